@@ -1,0 +1,438 @@
+"""Benchmark of the stage-boundary codec on GB300.
+
+One step is one pass of the whole boundary for one microbatch of the
+large-stream workload (T = 16 x 4096 tokens, d = 8192, k = 82, vocab 128256,
+Zipf(1.1) ids, 5% off-subspace energy):
+
+  sn_compress_fwd -> wire (device -> pinned host -> device) -> sn_decompress_fwd
+  sn_compress_bwd -> wire -> sn_decompress_bwd
+  sn_project_weight of the stage's attention out-projection W_o [8192, 8192]
+  (projected every iteration, Sec. 5)
+
+Inputs are resident in HBM when the timed region starts; L2 is flushed (a
+512 MiB write) before every timed step.  `value` is boundary tokens/s over the
+whole job; `e2e` is the same metric with the step's activation, ids and
+gradient copied in from pinned host memory and the reconstructed activation
+and gradient copied back, inside the timed region.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+WORKLOAD = "large"
+W_O_SHAPE = (8192, 8192)
+METRIC = "boundary tokens/sec (compress+decompress) and achieved HBM GB/s vs GB300 peak"
+L2_FLUSH_BYTES = 512 << 20
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0,
+                    help="target CPU time of the oracle baseline sample")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+# ---- algorithmic bytes (each unique embedding row counted once) --------------
+
+def algorithmic_bytes(T, d, k, n, u, m_cols, s=2):
+    """HBM bytes each call must move at minimum."""
+    emb = s * u * d + s * min(n, T) * d
+    return {
+        "sn_compress_fwd": s * T * d + emb + 4 * d * k + s * T * k,
+        "sn_decompress_fwd": s * T * d + emb + 4 * d * k + s * T * k,
+        "sn_compress_bwd": s * T * d + s * T * k + 4 * d * k,
+        "sn_decompress_bwd": s * T * d + s * T * k + 4 * d * k,
+        "sn_project_weight": 2 * s * d * m_cols,
+    }
+
+
+# ---- clocks ---------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    mx.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for name, val in zip(names, parts[5:9]):
+                    if val.lower() == "active":
+                        reasons.add(name)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# ---- distributed plumbing (independent replicas: no data-path collective) ----
+
+def dist_setup(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    pg = None
+    if world > 1:
+        import torch.distributed as dist
+        import torch
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+        pg = dist
+    return world, rank, local, pg
+
+
+def barrier(pg):
+    if pg is not None:
+        pg.barrier()
+
+
+def max_over_ranks(pg, value, device=None):
+    if pg is None:
+        return value
+    import torch
+    t = torch.tensor([float(value)], dtype=torch.float64,
+                     device=device if device is not None else "cpu")
+    pg.all_reduce(t, op=pg.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ---- CPU oracle baseline ---------------------------------------------------------
+
+def cpu_oracle_step_time(target_s, seed=7):
+    """Time the fp64 oracle on a bounded sample of the large-stream step and
+    scale it to a full step: S tokens through the four boundary calls, plus c
+    columns of W_o through the projection.  Returns (seconds per full step,
+    description of the sample)."""
+    import oracle as O
+    from paper_2506_01260_gb300 import workloads as W
+
+    wl = W.WORKLOADS[WORKLOAD]
+    orc = O.default()
+    rng = np.random.default_rng(seed)
+    d, k, n = wl.d, wl.k, wl.seq_len
+    U = W.orthonormal_basis(d, k, rng).astype(np.float32)
+
+    def boundary(S):
+        tok = W.to_bf16(0.02 * rng.standard_normal((S, d)))
+        pe = W.to_bf16(0.02 * rng.standard_normal((S, d)))
+        ids = np.arange(S, dtype=np.int32)
+        pos = np.arange(S, dtype=np.int32)
+        X = W.to_bf16(0.1 * rng.standard_normal((S, d)))
+        G = W.to_bf16(rng.standard_normal((S, d)))
+        t0 = time.perf_counter()
+        C, _, _ = orc.compress_fwd(X, ids, tok, U, S, pos_emb=pe, pos=pos)
+        orc.decompress_fwd(C, ids, tok, U, S, pos_emb=pe, pos=pos)
+        Cg, _, _ = orc.compress_bwd(G, U)
+        orc.decompress_bwd(Cg, U)
+        return time.perf_counter() - t0
+
+    def project(c):
+        Wc = W.to_bf16(0.02 * rng.standard_normal((d, c)))
+        t0 = time.perf_counter()
+        orc.project_weight(Wc, U)
+        return time.perf_counter() - t0
+
+    t_probe = boundary(8) / 8
+    S = int(max(8, min(wl.T, 0.85 * target_s / max(t_probe, 1e-9))))
+    tb = boundary(S)
+    p_probe = project(4) / 4
+    c = int(max(4, min(W_O_SHAPE[1], 0.15 * target_s / max(p_probe, 1e-9))))
+    tp = project(c)
+    step = tb * wl.T / S + tp * W_O_SHAPE[1] / c
+    desc = ("fp64 oracle, 1 thread: %d of %d tokens through compress_fwd+decompress_fwd+"
+            "compress_bwd+decompress_bwd (%.1f s) and %d of %d W_o columns through "
+            "project_weight (%.1f s), scaled to one full step" % (S, wl.T, tb, c, W_O_SHAPE[1], tp))
+    return step, desc, tb + tp
+
+
+def run_reference(args, world, rank):
+    """The oracle on the host cores, on the same workload, metric and unit."""
+    if rank != 0:
+        return
+    steps = []
+    desc = None
+    for i in range(args.warmup + args.steps):
+        st, desc, _ = cpu_oracle_step_time(max(1.0, args.cpu_seconds / 4), seed=100 + i)
+        if i >= args.warmup:
+            steps.append(st)
+    from paper_2506_01260_gb300 import workloads as W
+    T = W.WORKLOADS[WORKLOAD].T
+    ms = 1e3 * statistics.mean(steps)
+    value = T / (ms / 1e3)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": config_dict(),
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                         "sample": desc},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def config_dict():
+    return {"workload": "large stream: T=16x4096 tokens, d=8192, k=82, vocab 128256, bf16, "
+                        "Zipf(1.1) ids, 5% off-subspace energy; fwd+bwd boundary round trip "
+                        "through a pinned host wire, plus project_weight of W_o [8192, 8192]",
+            "T": 65536, "d": 8192, "k": 82, "vocab": 128256, "seq_len": 4096,
+            "w_o": list(W_O_SHAPE), "l2": "flushed before every timed step (512 MiB write)",
+            "parallelism": "independent replicas (one process per GPU)"}
+
+
+# ---- our arm -------------------------------------------------------------------------
+
+def run_ours(args, world, rank, local, pg):
+    import torch
+    from paper_2506_01260_gb300 import sn
+    from paper_2506_01260_gb300 import workloads as W
+
+    assert torch.cuda.is_available(), "bench needs a CUDA device"
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    wl = W.WORKLOADS[WORKLOAD]
+    T, d, k, n = wl.T, wl.d, wl.k, wl.seq_len
+    inp = W.generate_on_device(wl, dev, seed=wl.seed + rank)
+    u = W.unique_ids(inp["ids_host"])
+    g = torch.Generator(device=dev)
+    g.manual_seed(wl.seed + 1000 + rank)
+    Wo = (0.02 * torch.randn(*W_O_SHAPE, generator=g, device=dev)).to(torch.bfloat16)
+    basis = sn.Basis(inp["U"])
+    X, ids, tok, pe, G = inp["X"], inp["ids"], inp["tok_emb"], inp["pos_emb"], inp["G"]
+    C = torch.empty(T, k, dtype=torch.bfloat16, device=dev)
+    C_rx = torch.empty_like(C)
+    Cg = torch.empty_like(C)
+    Cg_rx = torch.empty_like(C)
+    Xr = torch.empty_like(X)
+    Gr = torch.empty_like(G)
+    Wp = torch.empty_like(Wo)
+    ws = torch.empty(max(16, sn.sn_project_weight_workspace(basis, torch.bfloat16, W_O_SHAPE[1])),
+                     dtype=torch.uint8, device=dev)
+    wire_f = torch.empty(C.numel() * 2, dtype=torch.uint8, pin_memory=True)
+    wire_b = torch.empty(C.numel() * 2, dtype=torch.uint8, pin_memory=True)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    names = ["sn_compress_fwd", "sn_decompress_fwd", "sn_compress_bwd", "sn_decompress_bwd",
+             "sn_project_weight"]
+
+    def step(ev=None):
+        # ev: list of 2 * len(names) + 1 events bracketing each kernel call
+        def mark(i):
+            if ev is not None:
+                ev[i].record(stream)
+        mark(0)
+        sn.sn_compress_fwd(basis, X, ids, tok, n, pos_emb=pe, out=C)
+        mark(1)
+        sn.sn_wire_send(C, wire_f)
+        sn.sn_wire_recv(wire_f, C_rx)
+        mark(2)
+        sn.sn_decompress_fwd(basis, C_rx, ids, tok, n, pos_emb=pe, out=Xr)
+        mark(3)
+        sn.sn_compress_bwd(basis, G, out=Cg)
+        mark(4)
+        sn.sn_wire_send(Cg, wire_b)
+        sn.sn_wire_recv(wire_b, Cg_rx)
+        mark(5)
+        sn.sn_decompress_bwd(basis, Cg_rx, out=Gr)
+        mark(6)
+        sn.sn_project_weight(basis, Wo, out=Wp, workspace=ws)
+        mark(7)
+
+    for _ in range(args.warmup):
+        flush.zero_()
+        step()
+    sn.sn_check_errors(basis)
+    torch.cuda.synchronize()
+
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(8)] for _ in range(args.steps)]
+    clocks = ClockSampler(local)
+    clocks.start()
+    barrier(pg)
+    torch.cuda.synchronize()
+    launches0 = sn.sn_launch_count()
+    wall0 = time.perf_counter()
+    for i in range(args.steps):
+        flush.zero_()
+        step(evs[i])
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - wall0
+    launches = sn.sn_launch_count() - launches0
+    barrier(pg)
+    clk = clocks.stop()
+    sn.sn_check_errors(basis)
+
+    per_step = [e[0].elapsed_time(e[7]) for e in evs]          # ms
+    seg = {  # ms per launch, averaged over the timed steps
+        "sn_compress_fwd": statistics.mean(e[0].elapsed_time(e[1]) for e in evs),
+        "wire_fwd": statistics.mean(e[1].elapsed_time(e[2]) for e in evs),
+        "sn_decompress_fwd": statistics.mean(e[2].elapsed_time(e[3]) for e in evs),
+        "sn_compress_bwd": statistics.mean(e[3].elapsed_time(e[4]) for e in evs),
+        "wire_bwd": statistics.mean(e[4].elapsed_time(e[5]) for e in evs),
+        "sn_decompress_bwd": statistics.mean(e[5].elapsed_time(e[6]) for e in evs),
+        "sn_project_weight": statistics.mean(e[6].elapsed_time(e[7]) for e in evs),
+    }
+    ms = statistics.mean(per_step)
+    ms = max_over_ranks(pg, ms, dev)
+    value = world * T / (ms / 1e3)
+
+    hbm, peak_kind = peaks()
+    ab = algorithmic_bytes(T, d, k, n, u, W_O_SHAPE[1])
+    kernels = {}
+    for name in names:
+        gbs = ab[name] / (seg[name] / 1e3) / 1e9
+        kernels[name] = {"ms": seg[name], "algorithmic_bytes": ab[name], "gbs": gbs,
+                         "frac": gbs / hbm}
+    dom = max(names, key=lambda nm: seg[nm])
+    traffic = None
+    tpath = os.path.join(ROOT, "profiles", "traffic.json")
+    if os.path.exists(tpath):
+        with open(tpath) as f:
+            traffic = json.load(f).get(dom)
+
+    # ---- end to end through the C ABI with host buffers ----
+    Xh = torch.empty(X.shape, dtype=X.dtype, pin_memory=True)
+    Gh = torch.empty(G.shape, dtype=G.dtype, pin_memory=True)
+    idsh = torch.empty(ids.shape, dtype=ids.dtype, pin_memory=True)
+    Xoh = torch.empty_like(Xh, pin_memory=True)
+    Goh = torch.empty_like(Gh, pin_memory=True)
+    Xh.copy_(X)
+    Gh.copy_(G)
+    idsh.copy_(ids)
+    h2d = Xh.numel() * 2 + Gh.numel() * 2 + idsh.numel() * 4
+    d2h = Xoh.numel() * 2 + Goh.numel() * 2
+
+    def e2e_step():
+        sn.sn_wire_recv(Xh, X)
+        sn.sn_wire_recv(idsh, ids)
+        sn.sn_wire_recv(Gh, G)
+        step()
+        sn.sn_wire_send(Xr, Xoh)
+        sn.sn_wire_send(Gr, Goh)
+
+    for _ in range(min(args.warmup, 3)):
+        flush.zero_()
+        e2e_step()
+    torch.cuda.synchronize()
+    e2e_ms = []
+    for _ in range(max(3, args.steps // 2)):
+        flush.zero_()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        e2e_step()
+        b.record(stream)
+        b.synchronize()
+        e2e_ms.append(a.elapsed_time(b))
+    sn.sn_check_errors(basis)
+    e2e = max_over_ranks(pg, statistics.mean(e2e_ms), dev)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        st, desc, _ = cpu_oracle_step_time(args.cpu_seconds)
+        cpu = {"value": T / st, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+               "sample": desc}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic", "config": config_dict(),
+            "roofline": {"bound": "hbm", "kernel": dom,
+                         "achieved": kernels[dom]["gbs"], "peak": hbm,
+                         "peak_kind": peak_kind, "unit": "GB/s",
+                         "frac": kernels[dom]["gbs"] / hbm, "traffic": traffic,
+                         "algorithmic_bytes_per_launch": ab[dom]},
+            "kernels": kernels,
+            "wire_ms": {"fwd": seg["wire_fwd"], "bwd": seg["wire_bwd"]},
+            "boundary_hbm_gbs": sum(ab[nm] for nm in names) / (
+                sum(seg[nm] for nm in names) / 1e3) / 1e9,
+            "e2e": {"value": world * T / (e2e / 1e3), "unit": "tokens/s",
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e},
+            "gpu_launches": launches,
+            "unique_ids": u,
+            "wall_s_timed_region": wall,
+            "clocks": clk,
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(line), flush=True)
+    basis.destroy()
+
+
+def main():
+    args = parse()
+    world, rank, local, pg = dist_setup(args)
+    if args.impl == "reference":
+        run_reference(args, world, rank)
+    else:
+        run_ours(args, world, rank, local, pg)
+    if pg is not None:
+        pg.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

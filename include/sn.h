@@ -1,0 +1,144 @@
+/*
+ * sn.h — C ABI of the GB300 (sm_103a) stage-boundary codec of Subspace Networks
+ * (arXiv 2506.01260).
+ *
+ * At a pipeline boundary the residual-stream activation X^{l+1} minus the
+ * locally recomputable embeddings lies in S = Col(U) once the projection
+ * weights' rows are confined to S (Sec. 4.2, Eq. recursive2; Sec. 4.3), so only
+ * its k coefficients on the orthonormal basis U cross the wire (Sec. 4.3.1,
+ * Eq. subtract), and the activation gradient is compressed the same way
+ * (Sec. 4.4, Eq. grad_compress).  The residual-writing weights are kept inside
+ * S by projecting them with P = U U^T (Sec. 4.3, Sec. 5, App. A).
+ *
+ * Conventions shared by every call
+ *   - Tensor pointers are device pointers (memory of the current CUDA device)
+ *     unless stated otherwise, owned by the caller, contiguous row-major, and
+ *     16-byte aligned (SN_ERR_ALIGNMENT otherwise).
+ *   - Calls are stream-ordered and asynchronous: they validate their
+ *     arguments, enqueue kernels on `stream` and return.  An argument error
+ *     returns synchronously and enqueues nothing.
+ *   - `dtype` applies to X, C, G, the embedding tables and W alike.  SN_BF16 runs
+ *     on the tensor cores (fp32 accumulation, one round-to-nearest-even to
+ *     bf16 at the end); SN_F32 runs in fp32 on the CUDA cores.  U is fp32 at
+ *     the ABI in both cases.
+ *   - Token t's position is pos[t] when `pos` is non-NULL, else t mod seq_len
+ *     (the batch is the row-major flattening of [b, seq_len]).  The positional
+ *     table has seq_len rows; when it is NULL nothing positional is subtracted
+ *     or added and `pos` is ignored.
+ *   - An id outside [0, vocab) (or a position outside [0, seq_len)) is never
+ *     clamped: that token's output row is written as zeros and the basis'
+ *     device error word records SN_ERR_BAD_ID, reported by sn_check_errors.
+ *   - Only sn_basis_create allocates (and sn_basis_destroy frees); no other
+ *     call allocates memory or falls back to the CPU.
+ *   - Every wait inside a kernel is bounded; a wait that expires records
+ *     SN_ERR_TIMEOUT in the error word and the kernel returns.
+ */
+#ifndef SN_H
+#define SN_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    SN_OK = 0,
+    SN_ERR_INVALID_ARG = 1,   /* bad size, NULL pointer, k > d, overlap, ... */
+    SN_ERR_ALIGNMENT = 2,     /* a pointer or leading dimension breaks the 16-byte rule */
+    SN_ERR_UNSUPPORTED = 3,   /* valid request this build does not implement */
+    SN_ERR_BAD_ID = 4,        /* asynchronous: an id or position was out of range */
+    SN_ERR_TIMEOUT = 5,       /* asynchronous: a bounded in-kernel wait expired */
+    SN_ERR_CUDA = 6           /* a CUDA runtime call failed */
+} sn_status;
+
+typedef enum { SN_BF16 = 0, SN_F32 = 1 } sn_dtype;
+
+/* Opaque basis handle: padded bf16/fp32 copies of U and the device error word. */
+typedef struct sn_basis *sn_basis_t;
+
+/* Same type as cudaStream_t (NULL = the legacy default stream). */
+typedef struct CUstream_st *sn_stream_t;
+
+/* Create a basis handle from U, a device fp32 [d, k] row-major matrix with
+ * orthonormal columns (Sec. 4.3: U_k, Col(U_k) = S; shared by every node and
+ * never sent per step).  U is copied; the caller keeps ownership of its
+ * buffer.  Requires 16 <= d, d % 8 == 0, 1 <= k <= min(d, 128).  Allocates the
+ * handle's device buffers, enqueues their initialisation on `stream` and
+ * synchronises `stream` before returning.  *out is set only on SN_OK. */
+sn_status sn_basis_create(const float *U, int32_t d, int32_t k, sn_basis_t *out,
+                          sn_stream_t stream);
+
+/* Free a handle (synchronises the device).  NULL is a no-op. */
+sn_status sn_basis_destroy(sn_basis_t basis);
+
+/* d and k of a handle (either pointer may be NULL). */
+sn_status sn_basis_shape(sn_basis_t basis, int32_t *d, int32_t *k);
+
+/* Forward compress, Sec. 4.3.1 Eq. (subtract):
+ *   C[t, :] = (X[t, :] - tok_emb[ids[t], :] - pos_emb[p(t), :]) U
+ * X: [T, d]; ids: int32 [T]; pos: int32 [T] or NULL; tok_emb: [vocab, d]
+ * (T_fixed, the fixed high-rank table); pos_emb: [seq_len, d] or NULL;
+ * C: [T, k], contiguous, no padding (the wire tensor, k/d of X). */
+sn_status sn_compress_fwd(sn_basis_t basis, sn_dtype dtype, const void *X, const int32_t *ids,
+                          const int32_t *pos, int64_t T, int32_t seq_len, const void *tok_emb,
+                          int64_t vocab, const void *pos_emb, void *C, sn_stream_t stream);
+
+/* Forward reconstruct, Sec. 4.3.1 (recovery at the next node):
+ *   X[t, :] = C[t, :] U^T + pos_emb[p(t), :] + tok_emb[ids[t], :]
+ * Arguments as in sn_compress_fwd with C an input [T, k] and X the output [T, d]. */
+sn_status sn_decompress_fwd(sn_basis_t basis, sn_dtype dtype, const void *C, const int32_t *ids,
+                            const int32_t *pos, int64_t T, int32_t seq_len, const void *tok_emb,
+                            int64_t vocab, const void *pos_emb, void *X, sn_stream_t stream);
+
+/* Gradient compress, Sec. 4.4 Eq. (grad_compress): C[t, :] = G[t, :] U.
+ * G: [T, d] activation gradient; C: [T, k]. */
+sn_status sn_compress_bwd(sn_basis_t basis, sn_dtype dtype, const void *G, int64_t T, void *C,
+                          sn_stream_t stream);
+
+/* Gradient recover, Sec. 4.4: G[t, :] = C[t, :] U^T.  C: [T, k]; G: [T, d]. */
+sn_status sn_decompress_bwd(sn_basis_t basis, sn_dtype dtype, const void *C, int64_t T, void *G,
+                            sn_stream_t stream);
+
+/* Bytes of device workspace sn_project_weight needs for `cols` columns. */
+sn_status sn_project_weight_workspace(sn_basis_t basis, sn_dtype dtype, int64_t cols,
+                                      size_t *bytes);
+
+/* Weight projection onto S, Sec. 4.3 (Row(W_p1), Row(W_p2) in S), Sec. 5
+ * (W_p1 every iteration, W_p2 at initialisation), App. A.  In the paper's
+ * layout W_p in R^{m x d} and W_p <- W_p U U^T; torch stores the transpose, so
+ * for W [rows = d, cols] with leading dimension ld (elements):
+ *   W_out = U (U^T W)     (A = U^T W is accumulated in fp32)
+ * W_out may equal W (in place); any other overlap is SN_ERR_INVALID_ARG.
+ * ld * element size must be a multiple of 16.  `workspace` is device memory of
+ * at least sn_project_weight_workspace bytes, used only during the call. */
+sn_status sn_project_weight(sn_basis_t basis, sn_dtype dtype, const void *W, int64_t rows,
+                            int64_t cols, int64_t ld, void *W_out, void *workspace,
+                            size_t workspace_bytes, sn_stream_t stream);
+
+/* Bytes on the wire for T tokens: T * k * element size (Sec. 4.3: k/d of X). */
+sn_status sn_wire_bytes(sn_basis_t basis, sn_dtype dtype, int64_t T, size_t *bytes);
+
+/* The emulated pipeline link (Sec. 8.1 sends the compressed tensor between
+ * stages; here the boundary is a pinned host buffer in one process).
+ * sn_wire_send copies `bytes` from device memory to host memory (pinned for
+ * asynchrony); sn_wire_recv copies host memory to device memory.  Both are
+ * stream-ordered cudaMemcpyAsync calls. */
+sn_status sn_wire_send(const void *src_device, void *dst_host, size_t bytes, sn_stream_t stream);
+sn_status sn_wire_recv(const void *src_host, void *dst_device, size_t bytes, sn_stream_t stream);
+
+/* Synchronise `stream`, then return and clear the basis' asynchronous error
+ * (SN_ERR_BAD_ID or SN_ERR_TIMEOUT; SN_OK if none was recorded). */
+sn_status sn_check_errors(sn_basis_t basis, sn_stream_t stream);
+
+/* Number of kernels this library has launched in this process. */
+uint64_t sn_launch_count(void);
+
+/* Static, human-readable name of a status code. */
+const char *sn_status_string(sn_status status);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* SN_H */

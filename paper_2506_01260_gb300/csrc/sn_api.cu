@@ -1,0 +1,323 @@
+// sn_api.cu — the C ABI (include/sn.h): argument validation, basis handles,
+// dispatch to the tensor-core (bf16) and CUDA-core (fp32) kernels, the wire
+// copies and the asynchronous error word.
+#include <atomic>
+#include <cstdlib>
+#include <new>
+
+#include "sn_internal.cuh"
+
+namespace sn {
+static std::atomic<uint64_t> g_launches{0};
+void count_launch(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
+}  // namespace sn
+
+namespace {
+
+constexpr int kMaxK = 128;
+constexpr int64_t kMaxRows = (int64_t)1 << 31;   // TMA coordinates are 32-bit
+
+bool aligned(const void *p, uintptr_t a) { return ((uintptr_t)p % a) == 0; }
+
+bool overlap(const void *a, size_t na, const void *b, size_t nb)
+{
+    const uintptr_t pa = (uintptr_t)a, pb = (uintptr_t)b;
+    return pa < pb + nb && pb < pa + na;
+}
+
+size_t esize(sn_dtype dt) { return dt == SN_BF16 ? 2 : 4; }
+
+sn_status cuda_status(cudaError_t e) { return e == cudaSuccess ? SN_OK : SN_ERR_CUDA; }
+
+// Common checks of a basis handle and dtype; the handle must live on the
+// current device.
+sn_status check_basis(sn_basis_t b, sn_dtype dt)
+{
+    if (!b || (dt != SN_BF16 && dt != SN_F32))
+        return SN_ERR_INVALID_ARG;
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess)
+        return SN_ERR_CUDA;
+    return dev == b->device ? SN_OK : SN_ERR_INVALID_ARG;
+}
+
+// Checks shared by the forward (embedding) calls.
+sn_status check_fwd(sn_basis_t b, sn_dtype dt, const void *in, const int32_t *ids,
+                    const int32_t *pos, int64_t T, int32_t seq_len, const void *tok,
+                    int64_t vocab, const void *pe, const void *out, size_t in_row,
+                    size_t out_row)
+{
+    sn_status st = check_basis(b, dt);
+    if (st != SN_OK)
+        return st;
+    if (T < 0 || T >= kMaxRows || seq_len <= 0 || vocab <= 0 || vocab >= kMaxRows)
+        return SN_ERR_INVALID_ARG;
+    if (T == 0)
+        return SN_OK;
+    if (!in || !ids || !tok || !out)
+        return SN_ERR_INVALID_ARG;
+    if (!aligned(in, 16) || !aligned(tok, 16) || !aligned(out, 16) || (pe && !aligned(pe, 16)) ||
+        !aligned(ids, 4) || (pos && !aligned(pos, 4)))
+        return SN_ERR_ALIGNMENT;
+    const size_t es = esize(dt);
+    if (overlap(in, (size_t)T * in_row * es, out, (size_t)T * out_row * es))
+        return SN_ERR_INVALID_ARG;
+    return SN_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *sn_status_string(sn_status s)
+{
+    switch (s) {
+    case SN_OK: return "SN_OK";
+    case SN_ERR_INVALID_ARG: return "SN_ERR_INVALID_ARG";
+    case SN_ERR_ALIGNMENT: return "SN_ERR_ALIGNMENT";
+    case SN_ERR_UNSUPPORTED: return "SN_ERR_UNSUPPORTED";
+    case SN_ERR_BAD_ID: return "SN_ERR_BAD_ID";
+    case SN_ERR_TIMEOUT: return "SN_ERR_TIMEOUT";
+    case SN_ERR_CUDA: return "SN_ERR_CUDA";
+    }
+    return "SN_ERR_UNKNOWN";
+}
+
+uint64_t sn_launch_count(void) { return sn::g_launches.load(std::memory_order_relaxed); }
+
+sn_status sn_basis_create(const float *U, int32_t d, int32_t k, sn_basis_t *out,
+                          sn_stream_t stream)
+{
+    if (!U || !out || d < 16 || d % 8 != 0 || k < 1 || k > d || k > kMaxK)
+        return SN_ERR_INVALID_ARG;
+    if (!aligned(U, 16))
+        return SN_ERR_ALIGNMENT;
+    sn_basis *b = new (std::nothrow) sn_basis();
+    if (!b)
+        return SN_ERR_CUDA;
+    if (cudaGetDevice(&b->device) != cudaSuccess) {
+        delete b;
+        return SN_ERR_CUDA;
+    }
+    b->d = d;
+    b->k = k;
+    b->n_pad = (k + 15) / 16 * 16;
+    b->k64 = (k + 63) / 64 * 64;
+    cudaError_t e = cudaSuccess;
+    if (e == cudaSuccess) e = cudaMalloc(&b->u32, sizeof(float) * (size_t)d * k);
+    if (e == cudaSuccess) e = cudaMalloc(&b->u32t, sizeof(float) * (size_t)d * k);
+    if (e == cudaSuccess) e = cudaMalloc(&b->ut16, sizeof(__nv_bfloat16) * (size_t)b->n_pad * d);
+    if (e == cudaSuccess) e = cudaMalloc(&b->up16, sizeof(__nv_bfloat16) * (size_t)d * b->k64);
+    if (e == cudaSuccess) e = cudaMalloc(&b->err, sizeof(unsigned int));
+    if (e == cudaSuccess) e = cudaMemsetAsync(b->err, 0, sizeof(unsigned int), stream);
+    if (e == cudaSuccess) e = sn::prepare_basis(*b, U, stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+    if (e != cudaSuccess) {
+        sn_basis_destroy(b);
+        return SN_ERR_CUDA;
+    }
+    *out = b;
+    return SN_OK;
+}
+
+sn_status sn_basis_destroy(sn_basis_t b)
+{
+    if (!b)
+        return SN_OK;
+    cudaError_t e = cudaSuccess, e2;
+    if ((e2 = cudaFree(b->u32)) != cudaSuccess) e = e2;
+    if ((e2 = cudaFree(b->u32t)) != cudaSuccess) e = e2;
+    if ((e2 = cudaFree(b->ut16)) != cudaSuccess) e = e2;
+    if ((e2 = cudaFree(b->up16)) != cudaSuccess) e = e2;
+    if ((e2 = cudaFree(b->err)) != cudaSuccess) e = e2;
+    delete b;
+    return cuda_status(e);
+}
+
+sn_status sn_basis_shape(sn_basis_t b, int32_t *d, int32_t *k)
+{
+    if (!b)
+        return SN_ERR_INVALID_ARG;
+    if (d) *d = b->d;
+    if (k) *k = b->k;
+    return SN_OK;
+}
+
+sn_status sn_compress_fwd(sn_basis_t b, sn_dtype dt, const void *X, const int32_t *ids,
+                          const int32_t *pos, int64_t T, int32_t seq_len, const void *tok,
+                          int64_t vocab, const void *pe, void *C, sn_stream_t stream)
+{
+    sn_status st = check_fwd(b, dt, X, ids, pos, T, seq_len, tok, vocab, pe, C, b ? b->d : 0,
+                             b ? b->k : 0);
+    if (st != SN_OK || T == 0)
+        return st;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (dt == SN_F32)
+        return cuda_status(sn::simt_compress<float>(*b, (const float *)X, ids, pos, T, seq_len,
+                                                    (const float *)tok, vocab, (const float *)pe,
+                                                    (float *)C, true, s));
+    return cuda_status(sn::simt_compress<__nv_bfloat16>(
+        *b, (const __nv_bfloat16 *)X, ids, pos, T, seq_len, (const __nv_bfloat16 *)tok, vocab,
+        (const __nv_bfloat16 *)pe, (__nv_bfloat16 *)C, true, s));
+}
+
+sn_status sn_decompress_fwd(sn_basis_t b, sn_dtype dt, const void *C, const int32_t *ids,
+                            const int32_t *pos, int64_t T, int32_t seq_len, const void *tok,
+                            int64_t vocab, const void *pe, void *X, sn_stream_t stream)
+{
+    sn_status st = check_fwd(b, dt, C, ids, pos, T, seq_len, tok, vocab, pe, X, b ? b->k : 0,
+                             b ? b->d : 0);
+    if (st != SN_OK || T == 0)
+        return st;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (dt == SN_F32)
+        return cuda_status(sn::simt_decompress<float>(*b, (const float *)C, ids, pos, T, seq_len,
+                                                      (const float *)tok, vocab,
+                                                      (const float *)pe, (float *)X, true, s));
+    return cuda_status(sn::simt_decompress<__nv_bfloat16>(
+        *b, (const __nv_bfloat16 *)C, ids, pos, T, seq_len, (const __nv_bfloat16 *)tok, vocab,
+        (const __nv_bfloat16 *)pe, (__nv_bfloat16 *)X, true, s));
+}
+
+sn_status sn_compress_bwd(sn_basis_t b, sn_dtype dt, const void *G, int64_t T, void *C,
+                          sn_stream_t stream)
+{
+    sn_status st = check_basis(b, dt);
+    if (st != SN_OK)
+        return st;
+    if (T < 0 || T >= kMaxRows)
+        return SN_ERR_INVALID_ARG;
+    if (T == 0)
+        return SN_OK;
+    if (!G || !C)
+        return SN_ERR_INVALID_ARG;
+    if (!aligned(G, 16) || !aligned(C, 16))
+        return SN_ERR_ALIGNMENT;
+    const size_t es = esize(dt);
+    if (overlap(G, (size_t)T * b->d * es, C, (size_t)T * b->k * es))
+        return SN_ERR_INVALID_ARG;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (dt == SN_F32)
+        return cuda_status(sn::simt_compress<float>(*b, (const float *)G, nullptr, nullptr, T, 1,
+                                                    nullptr, 1, nullptr, (float *)C, false, s));
+    return cuda_status(sn::simt_compress<__nv_bfloat16>(*b, (const __nv_bfloat16 *)G, nullptr,
+                                                        nullptr, T, 1, nullptr, 1, nullptr,
+                                                        (__nv_bfloat16 *)C, false, s));
+}
+
+sn_status sn_decompress_bwd(sn_basis_t b, sn_dtype dt, const void *C, int64_t T, void *G,
+                            sn_stream_t stream)
+{
+    sn_status st = check_basis(b, dt);
+    if (st != SN_OK)
+        return st;
+    if (T < 0 || T >= kMaxRows)
+        return SN_ERR_INVALID_ARG;
+    if (T == 0)
+        return SN_OK;
+    if (!G || !C)
+        return SN_ERR_INVALID_ARG;
+    if (!aligned(G, 16) || !aligned(C, 16))
+        return SN_ERR_ALIGNMENT;
+    const size_t es = esize(dt);
+    if (overlap(G, (size_t)T * b->d * es, C, (size_t)T * b->k * es))
+        return SN_ERR_INVALID_ARG;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (dt == SN_F32)
+        return cuda_status(sn::simt_decompress<float>(*b, (const float *)C, nullptr, nullptr, T,
+                                                      1, nullptr, 1, nullptr, (float *)G, false,
+                                                      s));
+    return cuda_status(sn::simt_decompress<__nv_bfloat16>(*b, (const __nv_bfloat16 *)C, nullptr,
+                                                          nullptr, T, 1, nullptr, 1, nullptr,
+                                                          (__nv_bfloat16 *)G, false, s));
+}
+
+sn_status sn_project_weight_workspace(sn_basis_t b, sn_dtype dt, int64_t cols, size_t *bytes)
+{
+    if (!b || !bytes || cols < 0 || (dt != SN_BF16 && dt != SN_F32))
+        return SN_ERR_INVALID_ARG;
+    *bytes = sizeof(float) * (size_t)b->k * (size_t)cols;
+    return SN_OK;
+}
+
+sn_status sn_project_weight(sn_basis_t b, sn_dtype dt, const void *W, int64_t rows,
+                            int64_t cols, int64_t ld, void *W_out, void *ws, size_t ws_bytes,
+                            sn_stream_t stream)
+{
+    sn_status st = check_basis(b, dt);
+    if (st != SN_OK)
+        return st;
+    if (rows != b->d || cols < 0 || ld < cols || cols >= kMaxRows || ld >= kMaxRows)
+        return SN_ERR_INVALID_ARG;
+    if (cols == 0)
+        return SN_OK;
+    if (!W || !W_out || !ws)
+        return SN_ERR_INVALID_ARG;
+    const size_t es = esize(dt);
+    if (!aligned(W, 16) || !aligned(W_out, 16) || !aligned(ws, 16) || (ld * es) % 16 != 0)
+        return SN_ERR_ALIGNMENT;
+    size_t need = 0;
+    sn_project_weight_workspace(b, dt, cols, &need);
+    if (ws_bytes < need)
+        return SN_ERR_INVALID_ARG;
+    const size_t wbytes = ((size_t)(rows - 1) * ld + cols) * es;
+    if (W != W_out && overlap(W, wbytes, W_out, wbytes))
+        return SN_ERR_INVALID_ARG;
+    if (overlap(ws, need, W, wbytes) || overlap(ws, need, W_out, wbytes))
+        return SN_ERR_INVALID_ARG;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (dt == SN_F32)
+        return cuda_status(sn::simt_project<float>(*b, (const float *)W, cols, ld, (float *)W_out,
+                                                   (float *)ws, s));
+    return cuda_status(sn::simt_project<__nv_bfloat16>(*b, (const __nv_bfloat16 *)W, cols, ld,
+                                                       (__nv_bfloat16 *)W_out, (float *)ws, s));
+}
+
+sn_status sn_wire_bytes(sn_basis_t b, sn_dtype dt, int64_t T, size_t *bytes)
+{
+    if (!b || !bytes || T < 0 || (dt != SN_BF16 && dt != SN_F32))
+        return SN_ERR_INVALID_ARG;
+    *bytes = (size_t)T * (size_t)b->k * esize(dt);
+    return SN_OK;
+}
+
+sn_status sn_wire_send(const void *src_device, void *dst_host, size_t bytes, sn_stream_t stream)
+{
+    if (bytes == 0)
+        return SN_OK;
+    if (!src_device || !dst_host)
+        return SN_ERR_INVALID_ARG;
+    return cuda_status(cudaMemcpyAsync(dst_host, src_device, bytes, cudaMemcpyDeviceToHost,
+                                       (cudaStream_t)stream));
+}
+
+sn_status sn_wire_recv(const void *src_host, void *dst_device, size_t bytes, sn_stream_t stream)
+{
+    if (bytes == 0)
+        return SN_OK;
+    if (!src_host || !dst_device)
+        return SN_ERR_INVALID_ARG;
+    return cuda_status(cudaMemcpyAsync(dst_device, src_host, bytes, cudaMemcpyHostToDevice,
+                                       (cudaStream_t)stream));
+}
+
+sn_status sn_check_errors(sn_basis_t b, sn_stream_t stream)
+{
+    if (!b)
+        return SN_ERR_INVALID_ARG;
+    unsigned int word = 0;
+    cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+    if (e == cudaSuccess)
+        e = cudaMemcpy(&word, b->err, sizeof word, cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess && word)
+        e = cudaMemset(b->err, 0, sizeof word);
+    if (e != cudaSuccess)
+        return SN_ERR_CUDA;
+    if (word & SN_EBIT_TIMEOUT)
+        return SN_ERR_TIMEOUT;
+    if (word & SN_EBIT_BAD_ID)
+        return SN_ERR_BAD_ID;
+    return SN_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,73 @@
+// sn_internal.cuh — types shared by the library's translation units.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "sn.h"
+
+// Bits of the per-basis device error word.
+enum : unsigned int {
+    SN_EBIT_BAD_ID = 1u,    // an id or position was out of range (row zeroed)
+    SN_EBIT_TIMEOUT = 2u,   // a bounded wait expired; the kernel gave up
+};
+
+// Padded copies of U kept by a basis handle.
+//   u32  [d, k]      fp32, as given (CUDA-core paths, row i = U[i, :])
+//   u32t [k, d]      fp32 transpose (CUDA-core reconstruction, coalesced in d)
+//   ut16 [n_pad, d]  bf16 U^T, rows >= k zero: B operand of the d -> k contraction
+//   up16 [d, k64]    bf16 U, columns >= k zero: operand of the k -> d expansion
+struct sn_basis {
+    int device;
+    int d, k;
+    int n_pad;   // k rounded up to 16 (MMA N of the compress contraction)
+    int k64;     // k rounded up to 64 (whole 128-byte swizzle atoms)
+    float *u32;
+    float *u32t;
+    __nv_bfloat16 *ut16;
+    __nv_bfloat16 *up16;
+    unsigned int *err;
+};
+
+namespace sn {
+
+// Counts every kernel the library launches (reported by sn_launch_count).
+void count_launch(int n = 1);
+
+// ---- CUDA-core kernels (fp32 path) -------------------------------------------
+template <typename E>
+cudaError_t simt_compress(const sn_basis &b, const E *X, const int32_t *ids, const int32_t *pos,
+                          int64_t T, int seq_len, const E *tok, int64_t vocab, const E *pe,
+                          E *C, bool gather, cudaStream_t s);
+template <typename E>
+cudaError_t simt_decompress(const sn_basis &b, const E *C, const int32_t *ids,
+                            const int32_t *pos, int64_t T, int seq_len, const E *tok,
+                            int64_t vocab, const E *pe, E *X, bool gather, cudaStream_t s);
+template <typename E>
+cudaError_t simt_project(const sn_basis &b, const E *W, int64_t cols, int64_t ld, E *W_out,
+                         float *A, cudaStream_t s);
+
+cudaError_t prepare_basis(sn_basis &b, const float *U, cudaStream_t s);
+
+// ---- tensor-core kernels (bf16 path, tcgen05 + TMA) -----------------------------
+struct TcArgs {
+    const __nv_bfloat16 *X;     // compress: X or G [T, d]; decompress: output X or G
+    const int32_t *ids;
+    const int32_t *pos;
+    const __nv_bfloat16 *tok;
+    const __nv_bfloat16 *pe;
+    __nv_bfloat16 *C;           // compress: output [T, k]; decompress: input
+    int64_t T;
+    int64_t vocab;
+    int seq_len;
+    bool gather;                // subtract / add the embeddings
+};
+cudaError_t tc_compress(const sn_basis &b, const TcArgs &a, cudaStream_t s);
+cudaError_t tc_decompress(const sn_basis &b, const TcArgs &a, __nv_bfloat16 *X_out,
+                          cudaStream_t s);
+cudaError_t tc_project(const sn_basis &b, const __nv_bfloat16 *W, int64_t cols, int64_t ld,
+                       __nv_bfloat16 *W_out, void *workspace, cudaStream_t s);
+size_t tc_project_workspace(const sn_basis &b, int64_t cols);
+
+}  // namespace sn

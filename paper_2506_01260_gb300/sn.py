@@ -1,0 +1,285 @@
+"""Thin Python binding of libsn.so (C ABI in include/sn.h).
+
+Argument marshalling only: each function checks tensor shapes and dtypes,
+passes raw pointers, sizes and the current CUDA stream to the C entry point of
+the same name, and raises SNError on a non-OK status.  Every step of the
+boundary runs in the library's kernels; torch supplies device memory, pinned
+host memory and streams.  There is no fallback: importing this module fails
+loudly when the library has not been built.
+"""
+import ctypes
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libsn.so")
+
+SN_OK, SN_ERR_INVALID_ARG, SN_ERR_ALIGNMENT, SN_ERR_UNSUPPORTED = 0, 1, 2, 3
+SN_ERR_BAD_ID, SN_ERR_TIMEOUT, SN_ERR_CUDA = 4, 5, 6
+SN_BF16, SN_F32 = 0, 1
+
+if not os.path.exists(LIB_PATH):
+    raise ImportError("libsn.so is not built: run `python -c \"import __graft_entry__ as g; "
+                      "g.build()\"` (needs nvcc)")
+
+_lib = ctypes.CDLL(LIB_PATH)
+_P = ctypes.c_void_p
+_I32, _I64, _SZ = ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t
+_ST = ctypes.c_int
+
+
+def _sig(name, args, res=_ST):
+    f = getattr(_lib, name)
+    f.argtypes = args
+    f.restype = res
+    return f
+
+
+_sig("sn_basis_create", [_P, _I32, _I32, ctypes.POINTER(_P), _P])
+_sig("sn_basis_destroy", [_P])
+_sig("sn_basis_shape", [_P, ctypes.POINTER(_I32), ctypes.POINTER(_I32)])
+_sig("sn_compress_fwd", [_P, _ST, _P, _P, _P, _I64, _I32, _P, _I64, _P, _P, _P])
+_sig("sn_decompress_fwd", [_P, _ST, _P, _P, _P, _I64, _I32, _P, _I64, _P, _P, _P])
+_sig("sn_compress_bwd", [_P, _ST, _P, _I64, _P, _P])
+_sig("sn_decompress_bwd", [_P, _ST, _P, _I64, _P, _P])
+_sig("sn_project_weight_workspace", [_P, _ST, _I64, ctypes.POINTER(_SZ)])
+_sig("sn_project_weight", [_P, _ST, _P, _I64, _I64, _I64, _P, _P, _SZ, _P])
+_sig("sn_wire_bytes", [_P, _ST, _I64, ctypes.POINTER(_SZ)])
+_sig("sn_wire_send", [_P, _P, _SZ, _P])
+_sig("sn_wire_recv", [_P, _P, _SZ, _P])
+_sig("sn_check_errors", [_P, _P])
+_sig("sn_launch_count", [], ctypes.c_uint64)
+_sig("sn_status_string", [_ST], ctypes.c_char_p)
+
+#: every function the C header declares (checked against include/sn.h by tests)
+EXPORTS = ["sn_basis_create", "sn_basis_destroy", "sn_basis_shape", "sn_compress_fwd",
+           "sn_decompress_fwd", "sn_compress_bwd", "sn_decompress_bwd",
+           "sn_project_weight_workspace", "sn_project_weight", "sn_wire_bytes", "sn_wire_send",
+           "sn_wire_recv", "sn_check_errors", "sn_launch_count", "sn_status_string"]
+
+
+class SNError(RuntimeError):
+    def __init__(self, status, where):
+        self.status = status
+        name = _lib.sn_status_string(status).decode()
+        super().__init__("%s returned %s" % (where, name))
+
+
+def _check(status, where):
+    if status != SN_OK:
+        raise SNError(status, where)
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else stream)
+
+
+def _dtype(t):
+    if t.dtype == torch.bfloat16:
+        return SN_BF16
+    if t.dtype == torch.float32:
+        return SN_F32
+    raise TypeError("unsupported dtype %s (bf16 or fp32)" % t.dtype)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _need(t, name, dtype=None, contiguous=True):
+    if not isinstance(t, torch.Tensor):
+        raise TypeError("%s must be a torch.Tensor" % name)
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError("%s must be %s, got %s" % (name, dtype, t.dtype))
+    if contiguous and not t.is_contiguous():
+        raise ValueError("%s must be contiguous" % name)
+
+
+class Basis:
+    """A basis handle: U [d, k] fp32 with orthonormal columns (Sec. 4.3)."""
+
+    def __init__(self, U, stream=None):
+        _need(U, "U", torch.float32)
+        if U.dim() != 2 or not U.is_cuda:
+            raise ValueError("U must be a 2-D CUDA tensor [d, k]")
+        h = _P()
+        _check(_lib.sn_basis_create(_ptr(U), U.shape[0], U.shape[1], ctypes.byref(h),
+                                    _stream(stream)), "sn_basis_create")
+        self._h = h
+        self.d, self.k = int(U.shape[0]), int(U.shape[1])
+        self.device = U.device
+
+    @property
+    def handle(self):
+        if self._h is None:
+            raise RuntimeError("basis destroyed")
+        return self._h
+
+    def destroy(self):
+        if getattr(self, "_h", None) is not None:
+            _check(_lib.sn_basis_destroy(self._h), "sn_basis_destroy")
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass
+
+
+def sn_basis_create(U, stream=None):
+    return Basis(U, stream)
+
+
+def sn_basis_destroy(basis):
+    basis.destroy()
+
+
+def sn_basis_shape(basis):
+    d, k = _I32(), _I32()
+    _check(_lib.sn_basis_shape(basis.handle, ctypes.byref(d), ctypes.byref(k)), "sn_basis_shape")
+    return int(d.value), int(k.value)
+
+
+def sn_compress_fwd(basis, X, ids, tok_emb, seq_len, pos_emb=None, pos=None, out=None,
+                    stream=None):
+    """C = (X - tok_emb[ids] - pos_emb[p]) U  (Sec. 4.3.1, Eq. subtract)."""
+    _need(X, "X")
+    _need(ids, "ids", torch.int32)
+    _need(tok_emb, "tok_emb", X.dtype)
+    if pos_emb is not None:
+        _need(pos_emb, "pos_emb", X.dtype)
+    if pos is not None:
+        _need(pos, "pos", torch.int32)
+    T = X.shape[0]
+    if X.shape != (T, basis.d) or ids.shape != (T,) or tok_emb.shape[1] != basis.d:
+        raise ValueError("shape mismatch")
+    if out is None:
+        out = torch.empty(T, basis.k, dtype=X.dtype, device=X.device)
+    _need(out, "out", X.dtype)
+    _check(_lib.sn_compress_fwd(basis.handle, _dtype(X), _ptr(X), _ptr(ids), _ptr(pos), T,
+                                seq_len, _ptr(tok_emb), tok_emb.shape[0], _ptr(pos_emb),
+                                _ptr(out), _stream(stream)), "sn_compress_fwd")
+    return out
+
+
+def sn_decompress_fwd(basis, C, ids, tok_emb, seq_len, pos_emb=None, pos=None, out=None,
+                      stream=None):
+    """X = C U^T + pos_emb[p] + tok_emb[ids]  (Sec. 4.3.1)."""
+    _need(C, "C")
+    _need(ids, "ids", torch.int32)
+    _need(tok_emb, "tok_emb", C.dtype)
+    if pos_emb is not None:
+        _need(pos_emb, "pos_emb", C.dtype)
+    if pos is not None:
+        _need(pos, "pos", torch.int32)
+    T = C.shape[0]
+    if C.shape != (T, basis.k) or ids.shape != (T,) or tok_emb.shape[1] != basis.d:
+        raise ValueError("shape mismatch")
+    if out is None:
+        out = torch.empty(T, basis.d, dtype=C.dtype, device=C.device)
+    _need(out, "out", C.dtype)
+    _check(_lib.sn_decompress_fwd(basis.handle, _dtype(C), _ptr(C), _ptr(ids), _ptr(pos), T,
+                                  seq_len, _ptr(tok_emb), tok_emb.shape[0], _ptr(pos_emb),
+                                  _ptr(out), _stream(stream)), "sn_decompress_fwd")
+    return out
+
+
+def sn_compress_bwd(basis, G, out=None, stream=None):
+    """C_g = G U  (Sec. 4.4, Eq. grad_compress)."""
+    _need(G, "G")
+    T = G.shape[0]
+    if G.shape != (T, basis.d):
+        raise ValueError("shape mismatch")
+    if out is None:
+        out = torch.empty(T, basis.k, dtype=G.dtype, device=G.device)
+    _need(out, "out", G.dtype)
+    _check(_lib.sn_compress_bwd(basis.handle, _dtype(G), _ptr(G), T, _ptr(out), _stream(stream)),
+           "sn_compress_bwd")
+    return out
+
+
+def sn_decompress_bwd(basis, C, out=None, stream=None):
+    """G = C_g U^T  (Sec. 4.4)."""
+    _need(C, "C")
+    T = C.shape[0]
+    if C.shape != (T, basis.k):
+        raise ValueError("shape mismatch")
+    if out is None:
+        out = torch.empty(T, basis.d, dtype=C.dtype, device=C.device)
+    _need(out, "out", C.dtype)
+    _check(_lib.sn_decompress_bwd(basis.handle, _dtype(C), _ptr(C), T, _ptr(out),
+                                  _stream(stream)), "sn_decompress_bwd")
+    return out
+
+
+def sn_project_weight_workspace(basis, dtype, cols):
+    n = _SZ()
+    code = SN_BF16 if dtype == torch.bfloat16 else SN_F32
+    _check(_lib.sn_project_weight_workspace(basis.handle, code, cols, ctypes.byref(n)),
+           "sn_project_weight_workspace")
+    return int(n.value)
+
+
+def sn_project_weight(basis, W, out=None, workspace=None, stream=None):
+    """W' = U (U^T W) for torch-layout W [d, cols] (Sec. 4.3, Sec. 5, App. A).
+    `out` may be W itself (in place).  W may be a row-strided view."""
+    _need(W, "W", contiguous=False)
+    if W.dim() != 2 or W.shape[0] != basis.d or W.stride(1) != 1:
+        raise ValueError("W must be [d, cols] with unit column stride")
+    rows, cols = W.shape
+    ld = W.stride(0)
+    if out is None:
+        out = torch.empty_like(W)
+    if out.stride() != W.stride() or out.shape != W.shape:
+        raise ValueError("out must have W's shape and strides")
+    need = sn_project_weight_workspace(basis, W.dtype, cols)
+    if workspace is None:
+        workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=W.device)
+    _check(_lib.sn_project_weight(basis.handle, _dtype(W), _ptr(W), rows, cols, ld, _ptr(out),
+                                  _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                  _stream(stream)), "sn_project_weight")
+    return out
+
+
+def sn_wire_bytes(basis, dtype, T):
+    n = _SZ()
+    code = SN_BF16 if dtype == torch.bfloat16 else SN_F32
+    _check(_lib.sn_wire_bytes(basis.handle, code, T, ctypes.byref(n)), "sn_wire_bytes")
+    return int(n.value)
+
+
+def sn_wire_send(src_device, dst_host, stream=None):
+    """Device tensor -> (pinned) host tensor of the same byte size."""
+    n = src_device.numel() * src_device.element_size()
+    if dst_host.numel() * dst_host.element_size() < n or dst_host.is_cuda:
+        raise ValueError("destination must be host memory of at least %d bytes" % n)
+    _check(_lib.sn_wire_send(_ptr(src_device), _ptr(dst_host), n, _stream(stream)),
+           "sn_wire_send")
+    return dst_host
+
+
+def sn_wire_recv(src_host, dst_device, stream=None):
+    """(Pinned) host tensor -> device tensor of the same byte size."""
+    n = src_host.numel() * src_host.element_size()
+    if dst_device.numel() * dst_device.element_size() < n or not dst_device.is_cuda:
+        raise ValueError("destination must be device memory of at least %d bytes" % n)
+    _check(_lib.sn_wire_recv(_ptr(src_host), _ptr(dst_device), n, _stream(stream)),
+           "sn_wire_recv")
+    return dst_device
+
+
+def sn_check_errors(basis, stream=None):
+    """Synchronise the stream; raise SNError if a bad id or a timeout was recorded."""
+    _check(_lib.sn_check_errors(basis.handle, _stream(stream)), "sn_check_errors")
+
+
+def sn_launch_count():
+    return int(_lib.sn_launch_count())
+
+
+def sn_status_string(status):
+    return _lib.sn_status_string(status).decode()

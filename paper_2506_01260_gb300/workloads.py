@@ -115,21 +115,25 @@ def token_ids(wl, rng, T=None):
     raise ValueError(wl.ids)
 
 
-def generate(wl, seed=None):
+def generate(wl, seed=None, T=None, dtype="bf16"):
     """All inputs of a workload as numpy arrays (host, exact bytes).
 
     Returns a dict: U64 (fp64 basis), U (fp32 basis as passed to the library),
-    tok_emb / pos_emb / X (bf16 bits), ids (int32), Z (fp64 coefficients
-    planted in X), and G (bf16 bits) when the workload has a gradient.
+    tok_emb / pos_emb / X (bf16 bits, or fp32 values when dtype == "f32"),
+    ids (int32), Z (fp64 coefficients planted in X), and G when the workload
+    has a gradient.  `T` overrides the token count (positions stay t mod n).
     Intended for sizes that fit comfortably in host memory.
     """
     rng = np.random.default_rng(wl.seed if seed is None else seed)
-    T, d, k, n = wl.T, wl.d, wl.k, wl.seq_len
+    T = wl.T if T is None else T
+    d, k, n = wl.d, wl.k, wl.seq_len
+    enc = to_bf16 if dtype == "bf16" else (lambda a: np.asarray(a).astype(np.float32))
+    dec = bf16_bits_to_f32 if dtype == "bf16" else (lambda a: a)
     U64 = orthonormal_basis(d, k, rng)
     U32 = U64.astype(np.float32)
-    tok = to_bf16(0.02 * rng.standard_normal((wl.vocab, d)))
-    pe = to_bf16(0.02 * rng.standard_normal((n, d)))
-    ids = token_ids(wl, rng)
+    tok = enc(0.02 * rng.standard_normal((wl.vocab, d)))
+    pe = enc(0.02 * rng.standard_normal((n, d)))
+    ids = token_ids(wl, rng, T)
     Z = rng.standard_normal((T, k))
     S = Z @ U64.T
     if wl.off_scale > 0 or wl.off_energy > 0:
@@ -141,11 +145,10 @@ def generate(wl, seed=None):
         else:
             N *= wl.off_scale
         S = S + N
-    E = bf16_bits_to_f32(tok)[ids].astype(np.float64) + \
-        np.tile(bf16_bits_to_f32(pe).astype(np.float64), (wl.batch, 1))
-    out = dict(U64=U64, U=U32, tok_emb=tok, pos_emb=pe, ids=ids, Z=Z, X=to_bf16(E + S))
+    E = dec(tok)[ids].astype(np.float64) + dec(pe)[np.arange(T) % n].astype(np.float64)
+    out = dict(U64=U64, U=U32, tok_emb=tok, pos_emb=pe, ids=ids, Z=Z, X=enc(E + S))
     if wl.grad:
-        out["G"] = to_bf16(rng.standard_normal((T, d)))
+        out["G"] = enc(rng.standard_normal((T, d)))
     return out
 
 

@@ -1,0 +1,305 @@
+"""GPU parity: every boundary call of the C ABI against the fp64 oracle.
+
+Bar (relative Frobenius error against the oracle's unrounded fp64 value):
+1e-2 for bf16 outputs, 1e-5 for fp32 outputs; bit-exact for gathers, wire byte
+counts and layouts.  Sizes span several 128-token tiles with ragged tails, k
+from 1 to 128, d from 16 to 8192; guard bands around every output catch
+out-of-bounds writes.
+"""
+import numpy as np
+import pytest
+import torch
+
+from gpu_util import TOL, dev, dtname, guarded, guards_intact, host, rel_fro, widen
+from paper_2506_01260_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+# (name, T, seq_len, d, k, vocab)
+CASES = [
+    ("ragged_d512_k20", 1000, 300, 512, 20, 3000),
+    ("short_d256_k8", 333, 128, 256, 8, 1024),
+    ("tiles_d1024_k41", 4173, 1024, 1024, 41, 5000),
+    ("kmax_d2048_k128", 300, 100, 2048, 128, 777),
+    ("wide_d8192_k82", 260, 4096, 8192, 82, 1000),
+    ("one_token_d64_k1", 1, 7, 64, 1, 5),
+    ("square_d16_k16", 70, 9, 16, 16, 33),
+    ("exact_tile_d256_k16", 256, 128, 256, 16, 300),
+]
+DTYPES = ["bf16", "f32"]
+
+
+def case_inputs(name, T, n, d, k, vocab, dtype, seed=0):
+    wl = W.Workload(name, 1, n, d, k, vocab, 1000 + seed + d + k, off_scale=1e-2, grad=True)
+    return W.generate(wl, T=T, dtype=dtype)
+
+
+@pytest.fixture(scope="module")
+def bases():
+    return {}
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
+@pytest.mark.parametrize("case", CASES, ids=[c[0] for c in CASES])
+def test_forward_round_trip(sn, oracle, case, dtype):
+    name, T, n, d, k, vocab = case
+    inp = case_inputs(name, T, n, d, k, vocab, dtype)
+    basis = sn.Basis(dev(inp["U"]))
+    X, tok, pe, ids = dev(inp["X"]), dev(inp["tok_emb"]), dev(inp["pos_emb"]), dev(inp["ids"])
+    tdt = X.dtype
+    fullC, C = guarded((T, k), tdt)
+    sn.sn_compress_fwd(basis, X, ids, tok, n, pos_emb=pe, out=C)
+    fullX, Xr = guarded((T, d), tdt)
+    sn.sn_decompress_fwd(basis, C, ids, tok, n, pos_emb=pe, out=Xr)
+    sn.sn_check_errors(basis)
+    assert guards_intact(fullC) and guards_intact(fullX)
+    _, C64, st = oracle.compress_fwd(inp["X"], inp["ids"], inp["tok_emb"], inp["U"], n,
+                                     pos_emb=inp["pos_emb"])
+    assert st == 0
+    assert rel_fro(host(C), C64) <= TOL[dtype]
+    _, X64, _ = oracle.decompress_fwd(host(C), inp["ids"], inp["tok_emb"], inp["U"], n,
+                                      pos_emb=inp["pos_emb"])
+    assert rel_fro(host(Xr), X64) <= TOL[dtype]
+    # wire layout: C is a contiguous [T, k] slab, T*k elements, nothing else
+    assert sn.sn_wire_bytes(basis, tdt, T) == T * k * (2 if dtype == "bf16" else 4)
+    basis.destroy()
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
+@pytest.mark.parametrize("case", CASES, ids=[c[0] for c in CASES])
+def test_backward_round_trip(sn, oracle, case, dtype):
+    name, T, n, d, k, vocab = case
+    inp = case_inputs(name, T, n, d, k, vocab, dtype)
+    basis = sn.Basis(dev(inp["U"]))
+    G = dev(inp["G"])
+    fullC, C = guarded((T, k), G.dtype)
+    sn.sn_compress_bwd(basis, G, out=C)
+    fullG, Gr = guarded((T, d), G.dtype)
+    sn.sn_decompress_bwd(basis, C, out=Gr)
+    sn.sn_check_errors(basis)
+    assert guards_intact(fullC) and guards_intact(fullG)
+    _, C64, _ = oracle.compress_bwd(inp["G"], inp["U"])
+    assert rel_fro(host(C), C64) <= TOL[dtype]
+    _, G64, _ = oracle.decompress_bwd(host(C), inp["U"])
+    assert rel_fro(host(Gr), G64) <= TOL[dtype]
+    basis.destroy()
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
+def test_explicit_positions_and_no_positional_table(sn, oracle, dtype):
+    T, n, d, k, vocab = 700, 50, 512, 24, 900
+    inp = case_inputs("pos", T, n, d, k, vocab, dtype, seed=5)
+    rng = np.random.default_rng(3)
+    pos = rng.integers(0, n, T).astype(np.int32)
+    basis = sn.Basis(dev(inp["U"]))
+    X, tok, pe, ids = dev(inp["X"]), dev(inp["tok_emb"]), dev(inp["pos_emb"]), dev(inp["ids"])
+    C = sn.sn_compress_fwd(basis, X, ids, tok, n, pos_emb=pe, pos=dev(pos))
+    Xr = sn.sn_decompress_fwd(basis, C, ids, tok, n, pos_emb=pe, pos=dev(pos))
+    C2 = sn.sn_compress_fwd(basis, X, ids, tok, n)
+    Xr2 = sn.sn_decompress_fwd(basis, C2, ids, tok, n)
+    sn.sn_check_errors(basis)
+    _, C64, _ = oracle.compress_fwd(inp["X"], inp["ids"], inp["tok_emb"], inp["U"], n,
+                                    pos_emb=inp["pos_emb"], pos=pos)
+    assert rel_fro(host(C), C64) <= TOL[dtype]
+    _, X64, _ = oracle.decompress_fwd(host(C), inp["ids"], inp["tok_emb"], inp["U"], n,
+                                      pos_emb=inp["pos_emb"], pos=pos)
+    assert rel_fro(host(Xr), X64) <= TOL[dtype]
+    _, C64, _ = oracle.compress_fwd(inp["X"], inp["ids"], inp["tok_emb"], inp["U"], n)
+    assert rel_fro(host(C2), C64) <= TOL[dtype]
+    _, X64, _ = oracle.decompress_fwd(host(C2), inp["ids"], inp["tok_emb"], inp["U"], n)
+    assert rel_fro(host(Xr2), X64) <= TOL[dtype]
+    basis.destroy()
+
+
+def test_gather_bit_exact(sn, oracle):
+    """C = 0 reconstructs round(T_fixed[ids] + P[pos]) bit-for-bit (bf16)."""
+    T, n, d, k, vocab = 1500, 256, 1024, 33, 4000
+    inp = case_inputs("gather", T, n, d, k, vocab, "bf16", seed=9)
+    basis = sn.Basis(dev(inp["U"]))
+    C0 = np.zeros((T, k), np.uint16)
+    Xr = sn.sn_decompress_fwd(basis, dev(C0), dev(inp["ids"]), dev(inp["tok_emb"]), n,
+                              pos_emb=dev(inp["pos_emb"]))
+    sn.sn_check_errors(basis)
+    Xo, _, _ = oracle.decompress_fwd(C0, inp["ids"], inp["tok_emb"], inp["U"], n,
+                                     pos_emb=inp["pos_emb"])
+    assert np.array_equal(host(Xr), Xo)
+    # without a positional table the output is the gathered row itself
+    Xr = sn.sn_decompress_fwd(basis, dev(C0), dev(inp["ids"]), dev(inp["tok_emb"]), n)
+    assert np.array_equal(host(Xr), inp["tok_emb"][inp["ids"]])
+    basis.destroy()
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
+def test_bad_ids_zero_rows_and_report(sn, oracle, dtype):
+    T, n, d, k, vocab = 400, 64, 256, 12, 500
+    inp = case_inputs("bad", T, n, d, k, vocab, dtype, seed=11)
+    ids = inp["ids"].copy()
+    ids[[5, 130, 399]] = [vocab, -3, 2**31 - 1]
+    basis = sn.Basis(dev(inp["U"]))
+    X, tok, pe = dev(inp["X"]), dev(inp["tok_emb"]), dev(inp["pos_emb"])
+    C = sn.sn_compress_fwd(basis, X, dev(ids), tok, n, pos_emb=pe)
+    with pytest.raises(sn.SNError) as e:
+        sn.sn_check_errors(basis)
+    assert e.value.status == sn.SN_ERR_BAD_ID
+    sn.sn_check_errors(basis)            # the error word was cleared
+    Ch = host(C)
+    assert np.all(widen(Ch[[5, 130, 399]]) == 0)
+    _, C64, st = oracle.compress_fwd(inp["X"], ids, inp["tok_emb"], inp["U"], n,
+                                     pos_emb=inp["pos_emb"])
+    assert st == 4
+    assert rel_fro(Ch, C64) <= TOL[dtype]
+    Xr = sn.sn_decompress_fwd(basis, C, dev(ids), tok, n, pos_emb=pe)
+    with pytest.raises(sn.SNError):
+        sn.sn_check_errors(basis)
+    assert np.all(widen(host(Xr)[[5, 130, 399]]) == 0)
+    # an explicit position outside [0, seq_len) is reported the same way
+    pos = (np.arange(T) % n).astype(np.int32)
+    pos[77] = n
+    C = sn.sn_compress_fwd(basis, X, dev(inp["ids"]), tok, n, pos_emb=pe, pos=dev(pos))
+    with pytest.raises(sn.SNError):
+        sn.sn_check_errors(basis)
+    assert np.all(widen(host(C)[77]) == 0)
+    basis.destroy()
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
+@pytest.mark.parametrize("d,k,cols,ld", [(512, 20, 1000, 1000), (256, 8, 300, 304),
+                                         (1024, 41, 77, 80), (2048, 128, 129, 136),
+                                         (16, 16, 8, 8)])
+def test_project_weight(sn, oracle, dtype, d, k, cols, ld):
+    rng = np.random.default_rng(d + k + cols)
+    U = W.orthonormal_basis(d, k, rng).astype(np.float32)
+    full = 0.02 * rng.standard_normal((d, ld))
+    Wh = W.to_bf16(full) if dtype == "bf16" else full.astype(np.float32)
+    basis = sn.Basis(dev(U))
+    Wd = dev(Wh)[:, :cols]
+    out_full = torch.full((d, ld), 7.0, dtype=Wd.dtype, device=Wd.device)
+    out = out_full[:, :cols]
+    sn.sn_project_weight(basis, Wd, out=out)
+    sn.sn_check_errors(basis)
+    _, W64, _ = oracle.project_weight(np.ascontiguousarray(Wh[:, :cols]), U)
+    assert rel_fro(host(out), W64) <= TOL[dtype]
+    if cols < ld:      # the padding columns beyond `cols` are untouched
+        assert bool((out_full[:, cols:] == 7.0).all())
+    # in place
+    Wd2 = Wd.clone()
+    sn.sn_project_weight(basis, Wd2, out=Wd2)
+    assert torch.equal(Wd2, out)
+    basis.destroy()
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
+def test_projection_identities(sn, dtype):
+    """P^2 = P and P U = U on the GPU output (Sec. 4.3; U^T U = I, App. A)."""
+    d, k, cols = 1024, 41, 512
+    rng = np.random.default_rng(5)
+    U64 = W.orthonormal_basis(d, k, rng)
+    basis = sn.Basis(dev(U64.astype(np.float32)))
+    Wh = W.to_bf16(0.02 * rng.standard_normal((d, cols))) if dtype == "bf16" else \
+        (0.02 * rng.standard_normal((d, cols))).astype(np.float32)
+    W1 = sn.sn_project_weight(basis, dev(Wh))
+    W2 = sn.sn_project_weight(basis, W1)
+    assert rel_fro(host(W2), widen(host(W1))) <= TOL[dtype]
+    B = rng.standard_normal((k, cols))
+    In = U64 @ B
+    Inh = W.to_bf16(In) if dtype == "bf16" else In.astype(np.float32)
+    Pin = sn.sn_project_weight(basis, dev(Inh))
+    assert rel_fro(host(Pin), widen(Inh)) <= 2 * TOL[dtype]
+    basis.destroy()
+
+
+def test_gradient_identity_app_a(sn):
+    """(G P) W' = G W' with W' = P W (App. A): projecting the incoming gradient
+    loses nothing below a projected residual-writing weight."""
+    d, k, m, T = 2048, 20, 512, 640
+    rng = np.random.default_rng(6)
+    U = W.orthonormal_basis(d, k, rng).astype(np.float32)
+    basis = sn.Basis(dev(U))
+    Wp = sn.sn_project_weight(basis, dev(W.to_bf16(0.02 * rng.standard_normal((d, m)))))
+    G = dev(W.to_bf16(rng.standard_normal((T, d))))
+    Gp = sn.sn_decompress_bwd(basis, sn.sn_compress_bwd(basis, G))
+    sn.sn_check_errors(basis)
+    lhs = Gp.float() @ Wp.float()
+    rhs = G.float() @ Wp.float()
+    err = float((lhs - rhs).norm() / rhs.norm())
+    assert err <= 1e-2, err
+    basis.destroy()
+
+
+def test_residual_closure(sn):
+    """With W' = P W, X = E + h W'^T lies in E + S and round-trips (Sec. 4.2-4.3)."""
+    T, n, d, k, vocab, m = 900, 300, 1024, 24, 2000, 256
+    rng = np.random.default_rng(12)
+    U = W.orthonormal_basis(d, k, rng).astype(np.float32)
+    basis = sn.Basis(dev(U))
+    Wp = sn.sn_project_weight(basis, dev(W.to_bf16(0.05 * rng.standard_normal((d, m)))))
+    h = torch.from_numpy(rng.standard_normal((T, m)).astype(np.float32)).cuda()
+    tok = dev(W.to_bf16(0.02 * rng.standard_normal((vocab, d))))
+    pe = dev(W.to_bf16(0.02 * rng.standard_normal((n, d))))
+    ids = dev(rng.integers(0, vocab, T).astype(np.int32))
+    pos = torch.arange(T, device="cuda") % n
+    Y = h @ Wp.float().T
+    X = (tok[ids].float() + pe[pos].float() + Y).to(torch.bfloat16)
+    Xr = sn.sn_decompress_fwd(basis, sn.sn_compress_fwd(basis, X, ids, tok, n, pos_emb=pe), ids,
+                              tok, n, pos_emb=pe)
+    sn.sn_check_errors(basis)
+    err = float((Xr.float() - X.float()).norm() / Y.norm())
+    assert err <= 1e-2, err
+    basis.destroy()
+
+
+def test_wire_round_trip(sn):
+    """compress -> pinned host wire -> device -> reconstruct equals the direct
+    reconstruction bit-for-bit; the wire carries exactly T*k*2 bytes."""
+    T, n, d, k, vocab = 2048, 512, 2048, 20, 3000
+    inp = case_inputs("wire", T, n, d, k, vocab, "bf16", seed=13)
+    basis = sn.Basis(dev(inp["U"]))
+    X, tok, pe, ids = dev(inp["X"]), dev(inp["tok_emb"]), dev(inp["pos_emb"]), dev(inp["ids"])
+    C = sn.sn_compress_fwd(basis, X, ids, tok, n, pos_emb=pe)
+    nbytes = sn.sn_wire_bytes(basis, torch.bfloat16, T)
+    assert nbytes == T * k * 2 == C.numel() * 2
+    wire = torch.empty(nbytes, dtype=torch.uint8, pin_memory=True)
+    sn.sn_wire_send(C, wire)
+    C_rx = torch.empty_like(C)
+    sn.sn_wire_recv(wire, C_rx)
+    X1 = sn.sn_decompress_fwd(basis, C_rx, ids, tok, n, pos_emb=pe)
+    X2 = sn.sn_decompress_fwd(basis, C, ids, tok, n, pos_emb=pe)
+    sn.sn_check_errors(basis)
+    assert torch.equal(C_rx, C)
+    assert torch.equal(X1, X2)
+    assert np.array_equal(wire.numpy(), host(C).view(np.uint8).reshape(-1))
+    basis.destroy()
+
+
+def test_zero_tokens_is_a_no_op(sn):
+    basis = sn.Basis(dev(W.orthonormal_basis(64, 4, np.random.default_rng(0)).astype(np.float32)))
+    X = torch.empty(0, 64, dtype=torch.bfloat16, device="cuda")
+    ids = torch.empty(0, dtype=torch.int32, device="cuda")
+    tok = torch.zeros(10, 64, dtype=torch.bfloat16, device="cuda")
+    C = sn.sn_compress_fwd(basis, X, ids, tok, 8)
+    assert C.shape == (0, 4)
+    G = sn.sn_decompress_bwd(basis, C)
+    assert G.shape == (0, 64)
+    sn.sn_check_errors(basis)
+    basis.destroy()
+
+
+def test_argument_errors(sn):
+    U = dev(W.orthonormal_basis(64, 4, np.random.default_rng(0)).astype(np.float32))
+    basis = sn.Basis(U)
+    X = torch.zeros(10, 64, dtype=torch.bfloat16, device="cuda")
+    tok = torch.zeros(10, 64, dtype=torch.bfloat16, device="cuda")
+    ids = torch.zeros(10, dtype=torch.int32, device="cuda")
+    with pytest.raises(sn.SNError) as e:      # misaligned X
+        raw = torch.zeros(10 * 64 + 1, dtype=torch.bfloat16, device="cuda")[1:].view(10, 64)
+        sn.sn_compress_fwd(basis, raw, ids, tok, 8)
+    assert e.value.status == sn.SN_ERR_ALIGNMENT
+    with pytest.raises(sn.SNError) as e:      # seq_len = 0
+        sn.sn_compress_fwd(basis, X, ids, tok, 0)
+    assert e.value.status == sn.SN_ERR_INVALID_ARG
+    with pytest.raises(sn.SNError) as e:      # output overlapping the input
+        sn.sn_compress_bwd(basis, X, out=X.view(-1)[:40].view(10, 4))
+    assert e.value.status == sn.SN_ERR_INVALID_ARG
+    with pytest.raises(sn.SNError):           # k > d
+        sn.Basis(torch.zeros(16, 17, device="cuda"))
+    basis.destroy()
