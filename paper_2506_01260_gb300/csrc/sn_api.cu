@@ -1,6 +1,6 @@
 // sn_api.cu — the C ABI (include/sn.h): argument validation, basis handles,
-// dispatch to the tensor-core (bf16) and CUDA-core (fp32) kernels, the wire
-// copies and the asynchronous error word.
+// the launch of each call's kernels (bf16: tcgen05 tensor-core kernels; fp32:
+// CUDA-core kernels), the wire copies and the asynchronous error word.
 #include <atomic>
 #include <cstdlib>
 #include <new>
@@ -156,9 +156,9 @@ sn_status sn_compress_fwd(sn_basis_t b, sn_dtype dt, const void *X, const int32_
         return cuda_status(sn::simt_compress<float>(*b, (const float *)X, ids, pos, T, seq_len,
                                                     (const float *)tok, vocab, (const float *)pe,
                                                     (float *)C, true, s));
-    return cuda_status(sn::simt_compress<__nv_bfloat16>(
-        *b, (const __nv_bfloat16 *)X, ids, pos, T, seq_len, (const __nv_bfloat16 *)tok, vocab,
-        (const __nv_bfloat16 *)pe, (__nv_bfloat16 *)C, true, s));
+    sn::TcArgs a{(const __nv_bfloat16 *)X, ids, pos, (const __nv_bfloat16 *)tok,
+                 (const __nv_bfloat16 *)pe, (__nv_bfloat16 *)C, T, vocab, seq_len, true};
+    return cuda_status(sn::tc_compress(*b, a, s));
 }
 
 sn_status sn_decompress_fwd(sn_basis_t b, sn_dtype dt, const void *C, const int32_t *ids,
@@ -174,9 +174,9 @@ sn_status sn_decompress_fwd(sn_basis_t b, sn_dtype dt, const void *C, const int3
         return cuda_status(sn::simt_decompress<float>(*b, (const float *)C, ids, pos, T, seq_len,
                                                       (const float *)tok, vocab,
                                                       (const float *)pe, (float *)X, true, s));
-    return cuda_status(sn::simt_decompress<__nv_bfloat16>(
-        *b, (const __nv_bfloat16 *)C, ids, pos, T, seq_len, (const __nv_bfloat16 *)tok, vocab,
-        (const __nv_bfloat16 *)pe, (__nv_bfloat16 *)X, true, s));
+    sn::TcArgs a{nullptr, ids, pos, (const __nv_bfloat16 *)tok, (const __nv_bfloat16 *)pe,
+                 (__nv_bfloat16 *)C, T, vocab, seq_len, true};
+    return cuda_status(sn::tc_decompress(*b, a, (__nv_bfloat16 *)X, s));
 }
 
 sn_status sn_compress_bwd(sn_basis_t b, sn_dtype dt, const void *G, int64_t T, void *C,
@@ -200,9 +200,9 @@ sn_status sn_compress_bwd(sn_basis_t b, sn_dtype dt, const void *G, int64_t T, v
     if (dt == SN_F32)
         return cuda_status(sn::simt_compress<float>(*b, (const float *)G, nullptr, nullptr, T, 1,
                                                     nullptr, 1, nullptr, (float *)C, false, s));
-    return cuda_status(sn::simt_compress<__nv_bfloat16>(*b, (const __nv_bfloat16 *)G, nullptr,
-                                                        nullptr, T, 1, nullptr, 1, nullptr,
-                                                        (__nv_bfloat16 *)C, false, s));
+    sn::TcArgs a{(const __nv_bfloat16 *)G, nullptr, nullptr, nullptr, nullptr,
+                 (__nv_bfloat16 *)C, T, 1, 1, false};
+    return cuda_status(sn::tc_compress(*b, a, s));
 }
 
 sn_status sn_decompress_bwd(sn_basis_t b, sn_dtype dt, const void *C, int64_t T, void *G,
@@ -227,16 +227,23 @@ sn_status sn_decompress_bwd(sn_basis_t b, sn_dtype dt, const void *C, int64_t T,
         return cuda_status(sn::simt_decompress<float>(*b, (const float *)C, nullptr, nullptr, T,
                                                       1, nullptr, 1, nullptr, (float *)G, false,
                                                       s));
-    return cuda_status(sn::simt_decompress<__nv_bfloat16>(*b, (const __nv_bfloat16 *)C, nullptr,
-                                                          nullptr, T, 1, nullptr, 1, nullptr,
-                                                          (__nv_bfloat16 *)G, false, s));
+    sn::TcArgs a{nullptr, nullptr, nullptr, nullptr, nullptr, (__nv_bfloat16 *)C, T, 1, 1,
+                 false};
+    return cuda_status(sn::tc_decompress(*b, a, (__nv_bfloat16 *)G, s));
 }
 
 sn_status sn_project_weight_workspace(sn_basis_t b, sn_dtype dt, int64_t cols, size_t *bytes)
 {
     if (!b || !bytes || cols < 0 || (dt != SN_BF16 && dt != SN_F32))
         return SN_ERR_INVALID_ARG;
-    *bytes = sizeof(float) * (size_t)b->k * (size_t)cols;
+    if (dt == SN_F32) {
+        *bytes = sizeof(float) * (size_t)b->k * (size_t)cols;
+        return SN_OK;
+    }
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev != b->device)
+        return SN_ERR_INVALID_ARG;
+    *bytes = sn::tc_project_workspace(*b, cols);
     return SN_OK;
 }
 
@@ -269,8 +276,8 @@ sn_status sn_project_weight(sn_basis_t b, sn_dtype dt, const void *W, int64_t ro
     if (dt == SN_F32)
         return cuda_status(sn::simt_project<float>(*b, (const float *)W, cols, ld, (float *)W_out,
                                                    (float *)ws, s));
-    return cuda_status(sn::simt_project<__nv_bfloat16>(*b, (const __nv_bfloat16 *)W, cols, ld,
-                                                       (__nv_bfloat16 *)W_out, (float *)ws, s));
+    return cuda_status(sn::tc_project(*b, (const __nv_bfloat16 *)W, cols, ld,
+                                      (__nv_bfloat16 *)W_out, ws, s));
 }
 
 sn_status sn_wire_bytes(sn_basis_t b, sn_dtype dt, int64_t T, size_t *bytes)

@@ -1,0 +1,372 @@
+// sn_tc_contract.cu — the d -> k contraction on the tcgen05 tensor cores.
+//
+//   CMODE_X  C[t, :] = (X[t, :] - T_fixed[id_t, :] - P[p_t, :]) U     Sec. 4.3.1, Eq. (subtract)
+//   CMODE_G  C[t, :] = G[t, :] U                                       Sec. 4.4, Eq. (grad_compress)
+//   CMODE_W  A^T[c, :] = W[:, c]^T U  (fp32 partials over a d-range)    first pass of W' = U (U^T W)
+//
+// Persistent CTAs of six warps walk 128-row tiles:
+//   warp 0     TMA producer: the X/G tile, the U^T chunk, and (CMODE_X) the
+//              gathered T_fixed rows (tile::gather4) and positional rows into
+//              a ring of shared-memory stages (X and U^T 128-byte swizzled,
+//              gathered rows unswizzled so every gather lands 128-byte aligned);
+//   warp 1     allocates TMEM and issues tcgen05.mma (M = 128, N = k padded
+//              to 16, K = 64 per stage) into a double-buffered fp32 accumulator;
+//   warps 2-5  CMODE_X: subtract the embeddings in fp32 and re-round to bf16
+//              in place (the MMA A operand); CMODE_W: transpose the W tile into
+//              the K-major A operand; then drain the accumulator (tcgen05.ld),
+//              round once to bf16 and store each warp's 32 rows of C as one
+//              contiguous slab.
+// Every wait is bounded; a wait that expires raises SN_EBIT_TIMEOUT and the
+// CTA drains its in-flight copies and MMAs, frees TMEM and returns.
+#include "sn_tc.cuh"
+#include "sn_tc_kernels.cuh"
+
+namespace sn {
+namespace tc {
+namespace {
+
+__device__ __forceinline__ uint32_t sub3(uint32_t x, uint32_t t, uint32_t p)
+{
+    return pack_bf16(bf_lo(x) - bf_lo(t) - bf_lo(p), bf_hi(x) - bf_hi(t) - bf_hi(p));
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(kThreads, 1) k_contract(const __grid_constant__ ContractParams p)
+{
+    extern __shared__ uint8_t smem_raw[];
+    uint32_t base = smem_u32(smem_raw);
+    const uint32_t pad = (1024u - (base & 1023u)) & 1023u;
+    base += pad;
+    uint8_t *smem = smem_raw + pad;
+
+    const int S = p.stages;
+    const ContractPlan pl = contract_plan(MODE, p.n_pad, p.k, p.has_pe, S);
+    const uint32_t bar = base + pl.bar_off;
+    const uint32_t full_b = bar, rr_b = bar + 8 * S, empty_b = bar + 16 * S;
+    const uint32_t accf_b = bar + 24 * S, acce_b = accf_b + 16, drain_b = acce_b + 16;
+    uint32_t *tmem_slot = (uint32_t *)(smem + pl.bar_off + 8 * (3 * S + 5));
+    volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t tmem_cols = 2 * p.acc_stride;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(full_b + 8 * s, 1);
+            mbar_init(rr_b + 8 * s, 4);
+            mbar_init(empty_b + 8 * s, 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(accf_b + 8 * b, 1);
+            mbar_init(acce_b + 8 * b, 4);
+        }
+        mbar_init(drain_b, 1);
+        *abort_flag = 0;
+        mbar_fence_init();
+    }
+    if (warp == 1)
+        tmem_alloc(smem_u32(tmem_slot), tmem_cols);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    const int nitems = p.ntiles * p.splits;
+    const int kc_total = p.nkc;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            tma_prefetch(&p.mapA);
+            tma_prefetch(&p.mapU);
+            if (MODE == CMODE_X) {
+                tma_prefetch(&p.mapTok);
+                if (p.has_pe) {
+                    tma_prefetch(&p.mapPE);
+                    tma_prefetch(&p.mapPEg);
+                }
+            }
+        }
+        uint32_t g = 0;
+        bool ok = true;
+        for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x) {
+            const int tile = item / p.splits, split = item % p.splits;
+            const int kc0 = split * p.kc_per_item;
+            const int kc1 = min(kc0 + p.kc_per_item, kc_total);
+            const int64_t r0 = MODE == CMODE_W ? (int64_t)tile * BM
+                                               : tile_row0(tile, p.reorder, p.batches, p.seq_len);
+            int rid[4] = {0, 0, 0, 0}, rps[4] = {0, 0, 0, 0};
+            bool pe_tile = false;
+            if (MODE == CMODE_X) {
+#pragma unroll
+                for (int r = 0; r < 4; ++r) {
+                    const int64_t t = r0 + 4 * lane + r;
+                    int id = 0, ps = 0;
+                    if (t < p.rows) {
+                        id = p.ids[t];
+                        if (id < 0 || id >= p.vocab)
+                            id = 0;                       // row zeroed by the epilogue
+                        if (p.has_pe) {
+                            ps = p.has_pos ? p.pos[t] : (int)(t % p.seq_len);
+                            if (ps < 0 || ps >= p.seq_len)
+                                ps = 0;
+                        }
+                    }
+                    rid[r] = id;
+                    rps[r] = ps;
+                }
+                pe_tile = p.has_pe && !p.has_pos && (r0 % p.seq_len) + BM <= p.seq_len;
+            }
+            for (int kc = kc0; kc < kc1; ++kc, ++g) {
+                const int s = g % S;
+                const uint32_t n = g / S;
+                if (!warp_wait(empty_b + 8 * s, (n & 1) ^ 1, abort_flag, p.err)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t st = base + s * pl.stage_bytes;
+                const uint32_t fb = full_b + 8 * s;
+                if (lane == 0)
+                    mbar_arrive_tx(fb, pl.tx_bytes);
+                __syncwarp();
+                if (lane == 0) {
+                    if (MODE == CMODE_W)
+                        tma_load_2d(st + pl.a_bytes + pl.u_bytes, &p.mapA, (int)r0, kc * BK, fb);
+                    else
+                        tma_load_2d(st, &p.mapA, kc * BK, (int)r0, fb);
+                    tma_load_2d(st + pl.a_bytes, &p.mapU, kc * BK, 0, fb);
+                    if (MODE == CMODE_X && pe_tile)
+                        tma_load_2d(st + pl.a_bytes + pl.u_bytes + pl.raw_bytes, &p.mapPE,
+                                    kc * BK, (int)(r0 % p.seq_len), fb);
+                }
+                if (MODE == CMODE_X) {
+                    tma_gather4(st + pl.a_bytes + pl.u_bytes + lane * 512, &p.mapTok, kc * BK,
+                                rid[0], rid[1], rid[2], rid[3], fb);
+                    if (p.has_pe && !pe_tile)
+                        tma_gather4(st + pl.a_bytes + pl.u_bytes + pl.raw_bytes + lane * 512,
+                                    &p.mapPEg, kc * BK, rps[0], rps[1], rps[2], rps[3], fb);
+                }
+            }
+        }
+        if (!ok && lane == 0) {   // let copies already issued land before the CTA exits
+            for (uint32_t i = g > (uint32_t)S ? g - S : 0; i < g; ++i)
+                drain_wait(full_b + 8 * (i % S), (i / S) & 1);
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16(BM, p.n_pad);
+            uint32_t g = 0, it = 0;
+            bool ok = true;
+            for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++it) {
+                const int split = item % p.splits;
+                const int kc0 = split * p.kc_per_item;
+                const int kc1 = min(kc0 + p.kc_per_item, kc_total);
+                const uint32_t b = it & 1, nb = it >> 1;
+                if (!mbar_wait(acce_b + 8 * b, (nb & 1) ^ 1, abort_flag, p.err)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t d_tmem = tmem + b * p.acc_stride;
+                for (int kc = kc0; kc < kc1; ++kc, ++g) {
+                    const int s = g % S;
+                    const uint32_t n = g / S;
+                    const uint32_t wb = (MODE == CMODE_G ? full_b : rr_b) + 8 * s;
+                    if (!mbar_wait(wb, n & 1, abort_flag, p.err)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t st = base + s * pl.stage_bytes;
+#pragma unroll
+                    for (int kk = 0; kk < BK / 16; ++kk)
+                        mma_bf16(d_tmem, sdesc_sw128(st + kk * 32),
+                                 sdesc_sw128(st + pl.a_bytes + kk * 32), idesc,
+                                 (kc > kc0 || kk > 0) ? 1u : 0u);
+                    mma_commit(empty_b + 8 * s);
+                }
+                if (ok)
+                    mma_commit(accf_b + 8 * b);
+            }
+            if (!ok) {   // wait for MMAs already issued before TMEM is freed
+                mma_commit(drain_b);
+                drain_wait(drain_b, 0);
+            }
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ compute warps
+        const int q = warp & 3;              // TMEM lane quarter of this warp
+        const int tt = threadIdx.x - 64;     // 0..127
+        const int row = 32 * q + lane;
+        uint32_t g = 0, it = 0;
+        bool ok = true;
+        for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++it) {
+            const int tile = item / p.splits, split = item % p.splits;
+            const int kc0 = split * p.kc_per_item;
+            const int kc1 = min(kc0 + p.kc_per_item, kc_total);
+            const int64_t r0 = MODE == CMODE_W ? (int64_t)tile * BM
+                                               : tile_row0(tile, p.reorder, p.batches, p.seq_len);
+            if (MODE != CMODE_G) {
+                for (int kc = kc0; kc < kc1; ++kc, ++g) {
+                    const int s = g % S;
+                    const uint32_t n = g / S;
+                    if (!warp_wait(full_b + 8 * s, n & 1, abort_flag, p.err)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t st = base + s * pl.stage_bytes;
+                    if (MODE == CMODE_X) {
+                        // X tile swizzled; gathered T_fixed / P rows unswizzled (128 B each)
+                        const uint32_t tb = st + pl.a_bytes + pl.u_bytes;
+                        const uint32_t pb = tb + pl.raw_bytes;
+#pragma unroll 4
+                        for (int u = 0; u < 8; ++u) {
+                            const int unit = tt + 128 * u;
+                            const uint32_t xo = sw128(unit >> 3, unit & 7);
+                            const uint32_t po = (uint32_t)unit * 16;
+                            const uint4 x = lds128(st + xo);
+                            const uint4 t = lds128(tb + po);
+                            const uint4 e = p.has_pe ? lds128(pb + po) : make_uint4(0, 0, 0, 0);
+                            sts128(st + xo, make_uint4(sub3(x.x, t.x, e.x), sub3(x.y, t.y, e.y),
+                                                       sub3(x.z, t.z, e.z), sub3(x.w, t.w, e.w)));
+                        }
+                    } else {   // CMODE_W: raw W tile [64 d][128 c] -> A operand [128 c][64 d]
+                        const uint32_t raw = st + pl.a_bytes + pl.u_bytes;
+#pragma unroll
+                        for (int c = 0; c < 8; ++c) {
+                            uint32_t w[4];
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) {
+                                unsigned short lo, hi;
+                                asm volatile("ld.shared.u16 %0, [%1];"
+                                             : "=h"(lo)
+                                             : "r"(raw + (8 * c + 2 * e) * 256 + tt * 2));
+                                asm volatile("ld.shared.u16 %0, [%1];"
+                                             : "=h"(hi)
+                                             : "r"(raw + (8 * c + 2 * e + 1) * 256 + tt * 2));
+                                w[e] = (uint32_t)lo | ((uint32_t)hi << 16);
+                            }
+                            sts128(st + sw128(tt, c), make_uint4(w[0], w[1], w[2], w[3]));
+                        }
+                    }
+                    fence_async_smem();
+                    __syncwarp();
+                    if (lane == 0)
+                        mbar_arrive(rr_b + 8 * s);
+                }
+                if (!ok)
+                    break;
+            }
+            // ---- epilogue: accumulator -> output
+            const uint32_t b = it & 1, nb = it >> 1;
+            if (!warp_wait(accf_b + 8 * b, nb & 1, abort_flag, p.err)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t taddr = tmem + b * p.acc_stride + ((uint32_t)(32 * q) << 16);
+            if (MODE == CMODE_W) {
+                const int64_t c = r0 + row;
+                float *dst = p.P + ((int64_t)split * p.rows + c) * p.n_pad;
+                for (int cc = 0; cc < p.n_pad / 16; ++cc) {
+                    float v[16];
+                    tmem_ld16(taddr + 16 * cc, v);
+                    tmem_ld_wait();
+                    if (c < p.rows) {
+#pragma unroll
+                        for (int j = 0; j < 16; j += 4)
+                            *(float4 *)(dst + 16 * cc + j) =
+                                make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+                    }
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0)
+                    mbar_arrive(acce_b + 8 * b);
+            } else {
+                const int64_t t = r0 + row;
+                bool bad = false;
+                if (MODE == CMODE_X && t < p.rows) {
+                    const int id = p.ids[t];
+                    bad = id < 0 || id >= p.vocab;
+                    if (p.has_pe && p.has_pos) {
+                        const int ps = p.pos[t];
+                        bad = bad || ps < 0 || ps >= p.seq_len;
+                    }
+                    if (bad)
+                        atomicOr(p.err, SN_EBIT_BAD_ID);
+                }
+                __nv_bfloat16 *cst = (__nv_bfloat16 *)(smem + (size_t)S * pl.stage_bytes);
+                __nv_bfloat16 *crow = cst + (size_t)row * p.k;
+                for (int cc = 0; cc < p.n_pad / 16; ++cc) {
+                    float v[16];
+                    tmem_ld16(taddr + 16 * cc, v);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) {
+                        const int col = 16 * cc + j;
+                        if (col < p.k)
+                            crow[col] = __float2bfloat16_rn(bad ? 0.f : v[j]);
+                    }
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0)
+                    mbar_arrive(acce_b + 8 * b);
+                // this warp's 32 rows are one contiguous slab of 32 * k bf16 in C
+                const int64_t wr0 = r0 + 32 * q;
+                const int64_t nrows = p.rows - wr0 < 32 ? p.rows - wr0 : 32;
+                if (nrows > 0) {
+                    const uint32_t src = smem_u32(cst + (size_t)32 * q * p.k);
+                    uint8_t *dst = (uint8_t *)(p.C + wr0 * p.k);
+                    const int nbytes = (int)nrows * p.k * 2;
+                    for (int v = lane; v < nbytes / 16; v += 32)
+                        *(uint4 *)(dst + 16 * v) = lds128(src + 16 * v);
+                    for (int e = (nbytes / 16) * 8 + lane; e < nbytes / 2; e += 32)
+                        ((__nv_bfloat16 *)dst)[e] = cst[(size_t)32 * q * p.k + e];
+                }
+                __syncwarp();
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, tmem_cols);
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_contract(int mode, const ContractParams &p, int grid, cudaStream_t s)
+{
+    const ContractPlan pl = contract_plan(mode, p.n_pad, p.k, p.has_pe, p.stages);
+    cudaError_t e;
+    if (mode == CMODE_X) {
+        e = cudaFuncSetAttribute(k_contract<CMODE_X>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 pl.total);
+        if (e == cudaSuccess)
+            k_contract<CMODE_X><<<grid, kThreads, pl.total, s>>>(p);
+    } else if (mode == CMODE_G) {
+        e = cudaFuncSetAttribute(k_contract<CMODE_G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 pl.total);
+        if (e == cudaSuccess)
+            k_contract<CMODE_G><<<grid, kThreads, pl.total, s>>>(p);
+    } else {
+        e = cudaFuncSetAttribute(k_contract<CMODE_W>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 pl.total);
+        if (e == cudaSuccess)
+            k_contract<CMODE_W><<<grid, kThreads, pl.total, s>>>(p);
+    }
+    if (e != cudaSuccess)
+        return e;
+    count_launch();
+    return cudaGetLastError();
+}
+
+}  // namespace tc
+}  // namespace sn

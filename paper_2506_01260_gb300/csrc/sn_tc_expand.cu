@@ -1,0 +1,383 @@
+// sn_tc_expand.cu — the k -> d expansion on the tcgen05 tensor cores.
+//
+//   decompress_fwd  X[t, :] = C[t, :] U^T + P[p_t, :] + T_fixed[id_t, :]   Sec. 4.3.1
+//   decompress_bwd  G[t, :] = C[t, :] U^T                                 Sec. 4.4
+//   project (b)     W'[i, :] = U[i, :] A   with A = U^T W from the first pass
+//
+// A work item is one 128-row tile and a run of 64-column output blocks.
+//   warp 0     TMA producer: per block, the 64 rows of the B operand (U, or
+//              A^T; 128-byte swizzled) and, for the reconstruction, the gathered
+//              T_fixed rows (tile::gather4) and positional rows (unswizzled);
+//              per item, the A operand rows when they come from a tensor map;
+//   warp 1     TMEM allocation and tcgen05.mma (M = 128, N = 64, K = k padded
+//              to 16) into a double-buffered fp32 accumulator;
+//   warps 2-5  per item, repack the item's C rows into the swizzled K-major A
+//              operand (zero-padded to the MMA K); per block, drain the
+//              accumulator, add the positional and token rows in fp32, round
+//              once to bf16 into shared memory (over the gathered rows), and
+//              TMA-store each warp's 32 rows (rows past the end are clipped by
+//              the tensor map).
+// Every wait is bounded (SN_EBIT_TIMEOUT); an aborting CTA drains its copies
+// and MMAs and frees TMEM before it returns.
+#include "sn_tc.cuh"
+#include "sn_tc_kernels.cuh"
+
+namespace sn {
+namespace tc {
+namespace {
+
+__device__ __forceinline__ uint32_t add3(float a0, float a1, uint32_t p, uint32_t t)
+{
+    return pack_bf16(a0 + bf_lo(p) + bf_lo(t), a1 + bf_hi(p) + bf_hi(t));
+}
+
+template <int AMODE, bool GATHER>
+__global__ void __launch_bounds__(kThreads, 1) k_expand(const __grid_constant__ ExpandParams p)
+{
+    extern __shared__ uint8_t smem_raw[];
+    uint32_t base = smem_u32(smem_raw);
+    const uint32_t pad = (1024u - (base & 1023u)) & 1023u;
+    base += pad;
+    uint8_t *smem = smem_raw + pad;
+
+    const int S = p.stages;
+    const ExpandPlan pl = expand_plan(GATHER, p.katoms, p.has_pe, S);
+    const uint32_t a_s = base;
+    const uint32_t bar = base + pl.bar_off;
+    const uint32_t full_b = bar, empty_b = bar + 8 * S;
+    const uint32_t accf_b = bar + 16 * S, acce_b = accf_b + 16;
+    const uint32_t afull_b = acce_b + 16, aempty_b = afull_b + 8, drain_b = aempty_b + 8;
+    uint32_t *tmem_slot = (uint32_t *)(smem + pl.bar_off + 8 * (2 * S + 7));
+    volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    constexpr uint32_t kTmemCols = 2 * BN;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(full_b + 8 * s, 1);
+            mbar_init(empty_b + 8 * s, 4);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(accf_b + 8 * b, 1);
+            mbar_init(acce_b + 8 * b, 4);
+        }
+        mbar_init(afull_b, AMODE == AMODE_REPACK ? 4 : 1);
+        mbar_init(aempty_b, 1);
+        mbar_init(drain_b, 1);
+        *abort_flag = 0;
+        mbar_fence_init();
+    }
+    if (warp == 1)
+        tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    const int nitems = p.ntiles * p.chunks;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            tma_prefetch(&p.mapB);
+            if (AMODE == AMODE_TMA)
+                tma_prefetch(&p.mapA);
+            if (GATHER) {
+                tma_prefetch(&p.mapTok);
+                if (p.has_pe) {
+                    tma_prefetch(&p.mapPE);
+                    tma_prefetch(&p.mapPEg);
+                }
+            }
+        }
+        uint32_t g = 0, it = 0;
+        bool ok = true;
+        for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++it) {
+            const int tile = item / p.chunks, ch = item % p.chunks;
+            const int blk0 = ch * p.bpi, blk1 = min(blk0 + p.bpi, p.nblk);
+            const int64_t r0 = tile_row0(tile, p.reorder, p.batches, p.seq_len);
+            if (AMODE == AMODE_TMA) {
+                if (!warp_wait(aempty_b, (it & 1) ^ 1, abort_flag, p.err)) {
+                    ok = false;
+                    break;
+                }
+                if (lane == 0) {
+                    mbar_arrive_tx(afull_b, pl.a_bytes);
+                    for (int a = 0; a < p.katoms; ++a)
+                        tma_load_2d(a_s + a * kTile, &p.mapA, a * 64, (int)r0, afull_b);
+                }
+                __syncwarp();
+            }
+            int rid[4] = {0, 0, 0, 0}, rps[4] = {0, 0, 0, 0};
+            bool pe_tile = false;
+            if (GATHER) {
+#pragma unroll
+                for (int r = 0; r < 4; ++r) {
+                    const int64_t t = r0 + 4 * lane + r;
+                    int id = 0, ps = 0;
+                    if (t < p.rows) {
+                        id = p.ids[t];
+                        if (id < 0 || id >= p.vocab)
+                            id = 0;                       // row zeroed by the epilogue
+                        if (p.has_pe) {
+                            ps = p.has_pos ? p.pos[t] : (int)(t % p.seq_len);
+                            if (ps < 0 || ps >= p.seq_len)
+                                ps = 0;
+                        }
+                    }
+                    rid[r] = id;
+                    rps[r] = ps;
+                }
+                pe_tile = p.has_pe && !p.has_pos && (r0 % p.seq_len) + BM <= p.seq_len;
+            }
+            for (int blk = blk0; blk < blk1; ++blk, ++g) {
+                const int s = g % S;
+                const uint32_t n = g / S;
+                if (!warp_wait(empty_b + 8 * s, (n & 1) ^ 1, abort_flag, p.err)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t st = base + pl.a_bytes + s * pl.stage_bytes;
+                const uint32_t fb = full_b + 8 * s;
+                if (lane == 0)
+                    mbar_arrive_tx(fb, pl.tx_bytes);
+                __syncwarp();
+                if (lane == 0) {
+                    for (int a = 0; a < p.katoms; ++a)
+                        tma_load_2d(st + a * (BN * 128), &p.mapB, a * 64, blk * BN, fb);
+                    if (GATHER && pe_tile)
+                        tma_load_2d(st + pl.b_bytes + kTile, &p.mapPE, blk * BN,
+                                    (int)(r0 % p.seq_len), fb);
+                }
+                if (GATHER) {
+                    tma_gather4(st + pl.b_bytes + lane * 512, &p.mapTok, blk * BN, rid[0], rid[1],
+                                rid[2], rid[3], fb);
+                    if (p.has_pe && !pe_tile)
+                        tma_gather4(st + pl.b_bytes + kTile + lane * 512, &p.mapPEg, blk * BN,
+                                    rps[0], rps[1], rps[2], rps[3], fb);
+                }
+            }
+        }
+        if (!ok && lane == 0) {
+            for (uint32_t i = g > (uint32_t)S ? g - S : 0; i < g; ++i)
+                drain_wait(full_b + 8 * (i % S), (i / S) & 1);
+            if (AMODE == AMODE_TMA && it > 0)
+                drain_wait(afull_b, (it - 1) & 1);
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16(BM, BN);
+            uint32_t g = 0, it = 0;
+            bool ok = true;
+            for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++it) {
+                const int ch = item % p.chunks;
+                const int blk0 = ch * p.bpi, blk1 = min(blk0 + p.bpi, p.nblk);
+                if (!mbar_wait(afull_b, it & 1, abort_flag, p.err)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                for (int blk = blk0; blk < blk1; ++blk, ++g) {
+                    const int s = g % S;
+                    const uint32_t n = g / S, b = g & 1, nb = g >> 1;
+                    if (!mbar_wait(full_b + 8 * s, n & 1, abort_flag, p.err) ||
+                        !mbar_wait(acce_b + 8 * b, (nb & 1) ^ 1, abort_flag, p.err)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t st = base + pl.a_bytes + s * pl.stage_bytes;
+                    for (int kk = 0; kk < p.kmma; ++kk) {
+                        const uint32_t a = kk >> 2, off = (kk & 3) * 32;
+                        mma_bf16(tmem + b * BN, sdesc_sw128(a_s + a * kTile + off),
+                                 sdesc_sw128(st + a * (BN * 128) + off), idesc, kk > 0 ? 1u : 0u);
+                    }
+                    mma_commit(accf_b + 8 * b);
+                }
+                if (ok)
+                    mma_commit(aempty_b);
+            }
+            if (!ok) {
+                mma_commit(drain_b);
+                drain_wait(drain_b, 0);
+            }
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ compute warps
+        const int q = warp & 3;
+        const int tt = threadIdx.x - 64;
+        const int row = 32 * q + lane;
+        uint32_t g = 0, it = 0;
+        bool ok = true;
+        for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++it) {
+            const int tile = item / p.chunks, ch = item % p.chunks;
+            const int blk0 = ch * p.bpi, blk1 = min(blk0 + p.bpi, p.nblk);
+            const int64_t r0 = tile_row0(tile, p.reorder, p.batches, p.seq_len);
+            if (AMODE == AMODE_REPACK) {
+                // A operand: rows r0 .. r0+127 of C, zero-padded to katoms * 64 columns
+                if (!warp_wait(aempty_b, (it & 1) ^ 1, abort_flag, p.err)) {
+                    ok = false;
+                    break;
+                }
+                const int64_t t = r0 + tt;
+                const unsigned short *crow = (const unsigned short *)p.C + t * p.k;
+                for (int a = 0; a < p.katoms; ++a) {
+#pragma unroll 2
+                    for (int c = 0; c < 8; ++c) {
+                        uint32_t w[4];
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const int j = a * 64 + c * 8 + 2 * e;
+                            uint32_t lo = 0, hi = 0;
+                            if (t < p.rows) {
+                                if (j < p.k)
+                                    lo = __ldg(crow + j);
+                                if (j + 1 < p.k)
+                                    hi = __ldg(crow + j + 1);
+                            }
+                            w[e] = lo | (hi << 16);
+                        }
+                        sts128(a_s + a * kTile + sw128(tt, c), make_uint4(w[0], w[1], w[2], w[3]));
+                    }
+                }
+                fence_async_smem();
+                __syncwarp();
+                if (lane == 0)
+                    mbar_arrive(afull_b);
+            }
+            bool bad = false;
+            if (GATHER) {
+                const int64_t t = r0 + row;
+                if (t < p.rows) {
+                    const int id = p.ids[t];
+                    bad = id < 0 || id >= p.vocab;
+                    if (p.has_pe && p.has_pos) {
+                        const int ps = p.pos[t];
+                        bad = bad || ps < 0 || ps >= p.seq_len;
+                    }
+                    if (bad && ch == 0)
+                        atomicOr(p.err, SN_EBIT_BAD_ID);
+                }
+            }
+            for (int blk = blk0; blk < blk1; ++blk, ++g) {
+                const int s = g % S;
+                const uint32_t n = g / S, b = g & 1, nb = g >> 1;
+                if (!warp_wait(accf_b + 8 * b, nb & 1, abort_flag, p.err)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                float v[BN];
+                const uint32_t taddr = tmem + b * BN + ((uint32_t)(32 * q) << 16);
+#pragma unroll
+                for (int i = 0; i < BN / 16; ++i)
+                    tmem_ld16(taddr + 16 * i, *(float(*)[16])(v + 16 * i));
+                tmem_ld_wait();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0)
+                    mbar_arrive(acce_b + 8 * b);
+                if (GATHER && !warp_wait(full_b + 8 * s, n & 1, abort_flag, p.err)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t slot = base + pl.a_bytes + s * pl.stage_bytes + pl.b_bytes;
+                const uint32_t pslot = slot + kTile;
+                if (GATHER) {
+                    // Gathered rows are unswizzled 128-byte rows, so a thread (one row)
+                    // walks its 16-byte chunks starting at chunk (row & 7): the 8 rows of
+                    // a quarter-warp then touch 8 different banks.  Rotate the
+                    // accumulator by the same amount so chunk c of v is chunk
+                    // (c + rot) & 7 of the row.
+                    const int rot = row & 7;
+#pragma unroll
+                    for (int sh = 1; sh <= 4; sh <<= 1) {
+                        const bool on = (rot & sh) != 0;
+                        float w[BN];
+#pragma unroll
+                        for (int i = 0; i < BN; ++i)
+                            w[i] = on ? v[(i + 8 * sh) & (BN - 1)] : v[i];
+#pragma unroll
+                        for (int i = 0; i < BN; ++i)
+                            v[i] = w[i];
+                    }
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) {
+                        const uint32_t off = (uint32_t)row * 128 + (((c + rot) & 7) << 4);
+                        const uint4 tv = lds128(slot + off);
+                        const uint4 pv = p.has_pe ? lds128(pslot + off) : make_uint4(0, 0, 0, 0);
+                        uint4 o = make_uint4(add3(v[8 * c + 0], v[8 * c + 1], pv.x, tv.x),
+                                             add3(v[8 * c + 2], v[8 * c + 3], pv.y, tv.y),
+                                             add3(v[8 * c + 4], v[8 * c + 5], pv.z, tv.z),
+                                             add3(v[8 * c + 6], v[8 * c + 7], pv.w, tv.w));
+                        if (bad)
+                            o = make_uint4(0, 0, 0, 0);
+                        sts128(slot + off, o);       // in place: the store map is unswizzled
+                    }
+                } else {
+#pragma unroll
+                    for (int c = 0; c < 8; ++c)      // swizzled staging, swizzled store map
+                        sts128(slot + sw128(row, c),
+                               make_uint4(pack_bf16(v[8 * c + 0], v[8 * c + 1]),
+                                          pack_bf16(v[8 * c + 2], v[8 * c + 3]),
+                                          pack_bf16(v[8 * c + 4], v[8 * c + 5]),
+                                          pack_bf16(v[8 * c + 6], v[8 * c + 7])));
+                }
+                fence_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                    if (r0 + 32 * q < p.rows) {
+                        tma_store_2d(&p.mapOut, slot + q * 4096, blk * BN, (int)(r0 + 32 * q));
+                        bulk_commit();
+                        bulk_wait_read0();
+                    }
+                    mbar_arrive(empty_b + 8 * s);
+                }
+                __syncwarp();
+            }
+        }
+        if (lane == 0)
+            bulk_wait_all0();
+        __syncwarp();
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_expand(int amode, bool gather, const ExpandParams &p, int grid, cudaStream_t s)
+{
+    const ExpandPlan pl = expand_plan(gather, p.katoms, p.has_pe, p.stages);
+    cudaError_t e;
+    if (amode == AMODE_REPACK && gather) {
+        e = cudaFuncSetAttribute(k_expand<AMODE_REPACK, true>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, pl.total);
+        if (e == cudaSuccess)
+            k_expand<AMODE_REPACK, true><<<grid, kThreads, pl.total, s>>>(p);
+    } else if (amode == AMODE_REPACK) {
+        e = cudaFuncSetAttribute(k_expand<AMODE_REPACK, false>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, pl.total);
+        if (e == cudaSuccess)
+            k_expand<AMODE_REPACK, false><<<grid, kThreads, pl.total, s>>>(p);
+    } else {
+        e = cudaFuncSetAttribute(k_expand<AMODE_TMA, false>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, pl.total);
+        if (e == cudaSuccess)
+            k_expand<AMODE_TMA, false><<<grid, kThreads, pl.total, s>>>(p);
+    }
+    if (e != cudaSuccess)
+        return e;
+    count_launch();
+    return cudaGetLastError();
+}
+
+}  // namespace tc
+}  // namespace sn

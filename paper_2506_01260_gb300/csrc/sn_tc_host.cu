@@ -1,0 +1,313 @@
+// sn_tc_host.cu — host side of the tensor-core (bf16) path: TMA tensor maps,
+// shared-memory stage planning, work splitting, and the launch sequences of
+// the boundary calls.
+#include <algorithm>
+#include <cstring>
+#include <mutex>
+
+#include "sn_tc_kernels.cuh"
+
+namespace sn {
+namespace tc {
+namespace {
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                  const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                  const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn()
+{
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = (EncodeTiledFn)f;
+    });
+    return fn;
+}
+
+// A 2-D bf16 tensor of `outer` rows x `inner` elements, `row_bytes` apart.
+bool map2d(CUtensorMap *m, const void *ptr, uint64_t inner, uint64_t outer, uint64_t row_bytes,
+           uint32_t box_inner, uint32_t box_outer, bool sw128)
+{
+    EncodeTiledFn fn = encode_fn();
+    if (!fn)
+        return false;
+    const cuuint64_t dims[2] = {inner, outer};
+    const cuuint64_t strides[1] = {row_bytes};
+    const cuuint32_t box[2] = {box_inner, box_outer};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides, box,
+              estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+              sw128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int sm_count(int device)
+{
+    static int cache[64] = {0};
+    if (device < 0 || device >= 64)
+        return 148;
+    if (cache[device] == 0) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, device) != cudaSuccess ||
+            n <= 0)
+            n = 148;
+        cache[device] = n;
+    }
+    return cache[device];
+}
+
+int pow2_at_least(int v, int lo)
+{
+    int p = lo;
+    while (p < v)
+        p *= 2;
+    return p;
+}
+
+int contract_stages(int mode, int n_pad, int k, int has_pe)
+{
+    int s = 8;
+    while (s > 2 && contract_plan(mode, n_pad, k, has_pe, s).total > kSmemLimit)
+        --s;
+    return s;
+}
+
+int expand_stages(bool gather, int katoms, int has_pe)
+{
+    int s = 6;
+    while (s > 2 && expand_plan(gather, katoms, has_pe, s).total > kSmemLimit)
+        --s;
+    return s;
+}
+
+// Tiles ordered position-block-major when every sequence of the batch shares
+// the same positional rows in whole 128-row blocks.
+void tile_order(int64_t T, int seq_len, bool has_pe, bool has_pos, int *reorder, int *batches)
+{
+    *reorder = 0;
+    *batches = 1;
+    if (has_pe && !has_pos && seq_len % BM == 0 && T % seq_len == 0 && T / seq_len > 1) {
+        *reorder = 1;
+        *batches = (int)(T / seq_len);
+    }
+}
+
+// Split `nblk` column blocks of `ntiles` row tiles into work items so that a
+// persistent grid of `sms` CTAs sees several items each.
+void split_blocks(int ntiles, int nblk, int sms, int *bpi, int *chunks)
+{
+    int want = (4 * sms + ntiles - 1) / ntiles;
+    want = std::max(1, std::min(want, nblk));
+    *bpi = (nblk + want - 1) / want;
+    *chunks = (nblk + *bpi - 1) / *bpi;
+}
+
+// d-range splits of the projection's first pass.
+void project_splits(int d, int64_t m, int sms, int *splits, int *kc_per)
+{
+    const int nkc = (d + BK - 1) / BK;
+    const int64_t ntiles = (m + BM - 1) / BM;
+    int want = (int)std::max<int64_t>(1, (2 * sms + ntiles - 1) / ntiles);
+    want = std::min(want, nkc);
+    *kc_per = (nkc + want - 1) / want;
+    *splits = (nkc + *kc_per - 1) / *kc_per;
+}
+
+size_t align256(size_t v) { return (v + 255) & ~(size_t)255; }
+
+__global__ void k_sum_partials(const float *__restrict__ P, int splits, int64_t m, int n_pad,
+                               int k, int k64, __nv_bfloat16 *__restrict__ At)
+{
+    const int64_t n = m * k64;
+    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n;
+         e += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t c = e / k64;
+        const int j = (int)(e % k64);
+        float s = 0.f;
+        if (j < k)
+            for (int sp = 0; sp < splits; ++sp)
+                s += P[((int64_t)sp * m + c) * n_pad + j];
+        At[e] = __float2bfloat16_rn(s);
+    }
+}
+
+int current_device()
+{
+    int d = 0;
+    cudaGetDevice(&d);
+    return d;
+}
+
+}  // namespace
+}  // namespace tc
+
+cudaError_t tc_compress(const sn_basis &b, const TcArgs &a, cudaStream_t s)
+{
+    using namespace tc;
+    ContractParams p;
+    std::memset(&p, 0, sizeof p);
+    const bool has_pe = a.gather && a.pe != nullptr;
+    bool ok = map2d(&p.mapA, a.X, b.d, a.T, (uint64_t)b.d * 2, BK, BM, true) &&
+              map2d(&p.mapU, b.ut16, b.d, b.n_pad, (uint64_t)b.d * 2, BK, b.n_pad, true);
+    if (ok && a.gather)
+        ok = map2d(&p.mapTok, a.tok, b.d, a.vocab, (uint64_t)b.d * 2, BK, 1, false);
+    else
+        p.mapTok = p.mapA;
+    if (ok && has_pe)
+        ok = map2d(&p.mapPE, a.pe, b.d, a.seq_len, (uint64_t)b.d * 2, BK, BM, false) &&
+             map2d(&p.mapPEg, a.pe, b.d, a.seq_len, (uint64_t)b.d * 2, BK, 1, false);
+    else
+        p.mapPE = p.mapPEg = p.mapA;
+    if (!ok)
+        return cudaErrorInvalidValue;
+    const int mode = a.gather ? CMODE_X : CMODE_G;
+    p.ids = a.ids;
+    p.pos = a.pos;
+    p.C = a.C;
+    p.err = b.err;
+    p.rows = a.T;
+    p.vocab = a.vocab;
+    p.seq_len = a.seq_len;
+    p.has_pe = has_pe;
+    p.has_pos = a.gather && a.pos != nullptr;
+    p.d = b.d;
+    p.k = b.k;
+    p.n_pad = b.n_pad;
+    p.acc_stride = pow2_at_least(b.n_pad, 32);
+    p.nkc = (b.d + BK - 1) / BK;
+    p.kc_per_item = p.nkc;
+    p.splits = 1;
+    p.ntiles = (int)((a.T + BM - 1) / BM);
+    tile_order(a.T, a.seq_len, has_pe, p.has_pos, &p.reorder, &p.batches);
+    p.stages = contract_stages(mode, b.n_pad, b.k, has_pe);
+    const int grid = std::min(p.ntiles, sm_count(current_device()));
+    return launch_contract(mode, p, grid, s);
+}
+
+cudaError_t tc_decompress(const sn_basis &b, const TcArgs &a, __nv_bfloat16 *X_out,
+                          cudaStream_t s)
+{
+    using namespace tc;
+    ExpandParams p;
+    std::memset(&p, 0, sizeof p);
+    const bool has_pe = a.gather && a.pe != nullptr;
+    // the reconstruction stages its output over the (unswizzled) gathered rows
+    bool ok = map2d(&p.mapB, b.up16, b.k64, b.d, (uint64_t)b.k64 * 2, 64, BN, true) &&
+              map2d(&p.mapOut, X_out, b.d, a.T, (uint64_t)b.d * 2, 64, 32, !a.gather);
+    p.mapA = p.mapB;
+    if (ok && a.gather)
+        ok = map2d(&p.mapTok, a.tok, b.d, a.vocab, (uint64_t)b.d * 2, 64, 1, false);
+    else
+        p.mapTok = p.mapB;
+    if (ok && has_pe)
+        ok = map2d(&p.mapPE, a.pe, b.d, a.seq_len, (uint64_t)b.d * 2, 64, BM, false) &&
+             map2d(&p.mapPEg, a.pe, b.d, a.seq_len, (uint64_t)b.d * 2, 64, 1, false);
+    else
+        p.mapPE = p.mapPEg = p.mapB;
+    if (!ok)
+        return cudaErrorInvalidValue;
+    const int sms = sm_count(current_device());
+    p.C = a.C;
+    p.ids = a.ids;
+    p.pos = a.pos;
+    p.err = b.err;
+    p.rows = a.T;
+    p.vocab = a.vocab;
+    p.seq_len = a.seq_len;
+    p.has_pe = has_pe;
+    p.has_pos = a.gather && a.pos != nullptr;
+    p.k = b.k;
+    p.katoms = b.k64 / 64;
+    p.kmma = b.n_pad / 16;
+    p.ncols = b.d;
+    p.nblk = (b.d + BN - 1) / BN;
+    p.ntiles = (int)((a.T + BM - 1) / BM);
+    split_blocks(p.ntiles, p.nblk, sms, &p.bpi, &p.chunks);
+    tile_order(a.T, a.seq_len, has_pe, p.has_pos, &p.reorder, &p.batches);
+    p.stages = expand_stages(a.gather, p.katoms, has_pe);
+    const int grid = std::min(p.ntiles * p.chunks, sms);
+    return launch_expand(AMODE_REPACK, a.gather, p, grid, s);
+}
+
+size_t tc_project_workspace(const sn_basis &b, int64_t cols)
+{
+    using namespace tc;
+    int splits, kc_per;
+    project_splits(b.d, cols, sm_count(current_device()), &splits, &kc_per);
+    return align256(sizeof(float) * (size_t)splits * cols * b.n_pad) +
+           align256(sizeof(__nv_bfloat16) * (size_t)cols * b.k64);
+}
+
+cudaError_t tc_project(const sn_basis &b, const __nv_bfloat16 *W, int64_t cols, int64_t ld,
+                       __nv_bfloat16 *W_out, void *workspace, cudaStream_t s)
+{
+    using namespace tc;
+    const int sms = sm_count(current_device());
+    int splits, kc_per;
+    project_splits(b.d, cols, sms, &splits, &kc_per);
+    float *P = (float *)workspace;
+    __nv_bfloat16 *At = (__nv_bfloat16 *)((char *)workspace +
+                                          align256(sizeof(float) * (size_t)splits * cols * b.n_pad));
+    // pass 1: fp32 partials of A^T = (U^T W)^T over d-ranges
+    ContractParams p;
+    std::memset(&p, 0, sizeof p);
+    bool ok = map2d(&p.mapA, W, cols, b.d, (uint64_t)ld * 2, BM, BK, false) &&
+              map2d(&p.mapU, b.ut16, b.d, b.n_pad, (uint64_t)b.d * 2, BK, b.n_pad, true);
+    p.mapTok = p.mapPE = p.mapPEg = p.mapA;
+    if (!ok)
+        return cudaErrorInvalidValue;
+    p.P = P;
+    p.err = b.err;
+    p.rows = cols;
+    p.vocab = 1;
+    p.seq_len = 1;
+    p.d = b.d;
+    p.k = b.k;
+    p.n_pad = b.n_pad;
+    p.acc_stride = pow2_at_least(b.n_pad, 32);
+    p.nkc = (b.d + BK - 1) / BK;
+    p.kc_per_item = kc_per;
+    p.splits = splits;
+    p.ntiles = (int)((cols + BM - 1) / BM);
+    p.stages = contract_stages(CMODE_W, b.n_pad, b.k, 0);
+    cudaError_t e = launch_contract(CMODE_W, p, std::min(p.ntiles * splits, sms), s);
+    if (e != cudaSuccess)
+        return e;
+    // pass 2: sum the partials, round A^T to bf16 [cols, k64] (zero-padded)
+    k_sum_partials<<<2 * sms, 256, 0, s>>>(P, splits, cols, b.n_pad, b.k, b.k64, At);
+    count_launch();
+    if ((e = cudaGetLastError()) != cudaSuccess)
+        return e;
+    // pass 3: W' = U A, written through the W' tensor map
+    ExpandParams q;
+    std::memset(&q, 0, sizeof q);
+    ok = map2d(&q.mapA, b.up16, b.k64, b.d, (uint64_t)b.k64 * 2, 64, BM, true) &&
+         map2d(&q.mapB, At, b.k64, cols, (uint64_t)b.k64 * 2, 64, BN, true) &&
+         map2d(&q.mapOut, W_out, cols, b.d, (uint64_t)ld * 2, 64, 32, true);
+    q.mapTok = q.mapPE = q.mapPEg = q.mapB;
+    if (!ok)
+        return cudaErrorInvalidValue;
+    q.err = b.err;
+    q.rows = b.d;
+    q.vocab = 1;
+    q.seq_len = 1;
+    q.k = b.k;
+    q.katoms = b.k64 / 64;
+    q.kmma = b.n_pad / 16;
+    q.ncols = (int)cols;
+    q.nblk = (int)((cols + BN - 1) / BN);
+    q.ntiles = (b.d + BM - 1) / BM;
+    split_blocks(q.ntiles, q.nblk, sms, &q.bpi, &q.chunks);
+    q.stages = expand_stages(false, q.katoms, 0);
+    return launch_expand(AMODE_TMA, false, q, std::min(q.ntiles * q.chunks, sms), s);
+}
+
+}  // namespace sn

@@ -1,0 +1,127 @@
+// sn_tc_kernels.cuh — parameter blocks and shared-memory plans of the
+// tensor-core kernels (shared by the kernels and their host launchers).
+#pragma once
+
+#include <cuda.h>
+#include <stdint.h>
+
+#include "sn_internal.cuh"
+
+namespace sn {
+namespace tc {
+
+constexpr int BM = 128;          // rows (tokens / W columns / d rows) per tile = MMA M
+constexpr int BK = 64;           // contraction chunk: one 128-byte swizzle row of bf16
+constexpr int BN = 64;           // output columns per block of the expansion kernel
+constexpr int kThreads = 192;    // warp 0 TMA producer, warp 1 MMA, warps 2..5 compute
+constexpr uint32_t kSmemLimit = 232448;   // 227 KB per CTA
+constexpr uint32_t kTile = BM * 128;      // one [128 x 64] bf16 swizzled tile
+
+// ---- contraction: out[r, :] = A[r, :] . U   (A = X - E, G, or W^T) -----------
+enum { CMODE_G = 0, CMODE_X = 1, CMODE_W = 2 };
+
+struct ContractParams {
+    CUtensorMap mapA;    // X or G [T, d] (SW128, box 64 x 128) | W [d, m] (plain, box 128 x 64)
+    CUtensorMap mapU;    // U^T padded [n_pad, d] (SW128, box 64 x n_pad)
+    CUtensorMap mapTok;  // T_fixed [vocab, d] (SW128, box 64 x 1, gather4)
+    CUtensorMap mapPE;   // P [seq_len, d] (SW128, box 64 x 128)
+    CUtensorMap mapPEg;  // P [seq_len, d] (SW128, box 64 x 1, gather4)
+    const int32_t *ids;
+    const int32_t *pos;
+    __nv_bfloat16 *C;    // [T, k] output (G, X modes)
+    float *P;            // [splits, rows, n_pad] fp32 partial output (W mode)
+    unsigned int *err;
+    int64_t rows;        // T, or m (columns of W)
+    int64_t vocab;
+    int seq_len, has_pe, has_pos;
+    int d, k, n_pad, acc_stride;
+    int nkc;             // 64-wide chunks of d
+    int kc_per_item;     // chunks per work item (all of them unless split)
+    int splits;          // work items per row tile (W mode)
+    int ntiles;          // row tiles
+    int reorder, batches;
+    int stages;
+};
+
+struct ContractPlan {
+    uint32_t a_bytes, u_bytes, raw_bytes, pe_bytes, stage_bytes, cst_bytes, bar_off, total;
+    uint32_t tx_bytes;
+};
+
+__host__ __device__ inline ContractPlan contract_plan(int mode, int n_pad, int k, int has_pe,
+                                                      int stages)
+{
+    ContractPlan p;
+    p.a_bytes = kTile;
+    p.u_bytes = (uint32_t)n_pad * 128;
+    p.raw_bytes = (mode == CMODE_X || mode == CMODE_W) ? kTile : 0;   // T_fixed rows | raw W
+    p.pe_bytes = (mode == CMODE_X && has_pe) ? kTile : 0;
+    p.stage_bytes = p.a_bytes + p.u_bytes + p.raw_bytes + p.pe_bytes;
+    p.cst_bytes = (mode == CMODE_W) ? 0 : (((uint32_t)BM * k * 2 + 1023) & ~1023u);
+    p.bar_off = (uint32_t)stages * p.stage_bytes + p.cst_bytes;
+    p.total = p.bar_off + 8 * (3 * stages + 5) + 16 + 1024;   // + alignment slack
+    p.tx_bytes = (mode == CMODE_W) ? p.raw_bytes + p.u_bytes
+                                   : p.a_bytes + p.u_bytes + p.raw_bytes + p.pe_bytes;
+    return p;
+}
+
+// ---- expansion: out[r, n0:n0+64] = A[r, :] . B[n0:n0+64, :]^T (+ gathered rows) ------
+enum { AMODE_REPACK = 0, AMODE_TMA = 1 };
+
+struct ExpandParams {
+    CUtensorMap mapA;    // A by TMA: U padded [d, k64] (SW128, box 64 x 128)
+    CUtensorMap mapB;    // B rows: U padded [d, k64] | A^T [m, k64] (SW128, box 64 x 64)
+    CUtensorMap mapOut;  // output [rows, ncols] (SW128, box 64 x 32)
+    CUtensorMap mapTok;  // T_fixed (SW128, box 64 x 1, gather4)
+    CUtensorMap mapPE;   // P (SW128, box 64 x 128)
+    CUtensorMap mapPEg;  // P (SW128, box 64 x 1, gather4)
+    const __nv_bfloat16 *C;   // A by repacking: [rows, k]
+    const int32_t *ids;
+    const int32_t *pos;
+    unsigned int *err;
+    int64_t rows;        // T, or d
+    int64_t vocab;
+    int seq_len, has_pe, has_pos;
+    int k, katoms, kmma;
+    int ncols, nblk, bpi, chunks, ntiles;
+    int reorder, batches;
+    int stages;
+};
+
+struct ExpandPlan {
+    uint32_t a_bytes, b_bytes, out_bytes, pe_bytes, stage_bytes, bar_off, total, tx_bytes;
+};
+
+__host__ __device__ inline ExpandPlan expand_plan(bool gather, int katoms, int has_pe,
+                                                  int stages)
+{
+    ExpandPlan p;
+    p.a_bytes = (uint32_t)katoms * kTile;
+    p.b_bytes = (uint32_t)katoms * BN * 128;
+    p.out_bytes = kTile;                           // T_fixed rows, overwritten by the output
+    p.pe_bytes = (gather && has_pe) ? kTile : 0;
+    p.stage_bytes = p.b_bytes + p.out_bytes + p.pe_bytes;
+    p.bar_off = p.a_bytes + (uint32_t)stages * p.stage_bytes;
+    p.total = p.bar_off + 8 * (2 * stages + 7) + 16 + 1024;
+    p.tx_bytes = p.b_bytes + (gather ? p.out_bytes + p.pe_bytes : 0);
+    return p;
+}
+
+// Row tile -> first row.  With `reorder`, tiles run position-block-major so the
+// b sequences of a batch that share positional rows are processed together
+// and the positional table is read from HBM once.
+__host__ __device__ inline int64_t tile_row0(int tile, int reorder, int batches, int seq_len)
+{
+    if (reorder) {
+        const int b = tile % batches, pt = tile / batches;
+        return (int64_t)b * seq_len + (int64_t)pt * BM;
+    }
+    return (int64_t)tile * BM;
+}
+
+// ---- host side -----------------------------------------------------------------------
+cudaError_t launch_contract(int mode, const ContractParams &p, int grid, cudaStream_t s);
+cudaError_t launch_expand(int amode, bool gather, const ExpandParams &p, int grid, cudaStream_t s);
+
+}  // namespace tc
+}  // namespace sn
