@@ -33,6 +33,9 @@ sys.path.insert(0, ROOT)
 
 WORKLOAD = "large"
 W_O_SHAPE = (8192, 8192)
+# smaller cases with the same step, for profiling (the default is the large stream)
+PROFILE_WORKLOADS = {"large": ("large", (8192, 8192)), "8b": ("8b", (4096, 4096)),
+                     "1b": ("1b", (2048, 2048))}
 METRIC = "boundary tokens/sec (compress+decompress) and achieved HBM GB/s vs GB300 peak"
 L2_FLUSH_BYTES = 512 << 20
 
@@ -40,12 +43,15 @@ L2_FLUSH_BYTES = 512 << 20
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
-    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=300)
+    ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="target CPU time of the oracle baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--workload", choices=sorted(PROFILE_WORKLOADS), default=WORKLOAD,
+                    help="large (default, the benchmark) or a smaller case for profiling")
     return ap.parse_args()
 
 
@@ -90,7 +96,7 @@ class ClockSampler:
             os.close(fd)
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.FIELDS,
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "100"],
                 stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
         except (OSError, FileNotFoundError):
             self.proc = None
@@ -225,7 +231,7 @@ def run_reference(args, world, rank):
         "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": config_dict(),
+        "data": "synthetic", "config": config_dict(args.workload),
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
                          "sample": desc},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
@@ -234,12 +240,21 @@ def run_reference(args, world, rank):
     print(json.dumps(line), flush=True)
 
 
-def config_dict():
-    return {"workload": "large stream: T=16x4096 tokens, d=8192, k=82, vocab 128256, bf16, "
-                        "Zipf(1.1) ids, 5% off-subspace energy; fwd+bwd boundary round trip "
-                        "through a pinned host wire, plus project_weight of W_o [8192, 8192]",
-            "T": 65536, "d": 8192, "k": 82, "vocab": 128256, "seq_len": 4096,
-            "w_o": list(W_O_SHAPE), "l2": "flushed before every timed step (512 MiB write)",
+def config_dict(workload=WORKLOAD):
+    from paper_2506_01260_gb300 import workloads as W
+    wname, wo = PROFILE_WORKLOADS[workload]
+    wl = W.WORKLOADS[wname]
+    if workload == "large":
+        desc = ("large stream: T=16x4096 tokens, d=8192, k=82, vocab 128256, bf16, Zipf(1.1) "
+                "ids, 5% off-subspace energy; fwd+bwd boundary round trip through a pinned "
+                "host wire, plus project_weight of W_o [8192, 8192]")
+    else:
+        desc = ("%s-class: T=%dx%d tokens, d=%d, k=%d, vocab %d, bf16; fwd+bwd boundary round "
+                "trip through a pinned host wire, plus project_weight of W_o [%d, %d]"
+                % (wname.upper(), wl.batch, wl.seq_len, wl.d, wl.k, wl.vocab, wo[0], wo[1]))
+    return {"workload": desc, "T": wl.T, "d": wl.d, "k": wl.k, "vocab": wl.vocab,
+            "seq_len": wl.seq_len, "w_o": list(wo),
+            "l2": "flushed before every timed step (512 MiB write)",
             "parallelism": "independent replicas (one process per GPU)"}
 
 
@@ -253,13 +268,14 @@ def run_ours(args, world, rank, local, pg):
     assert torch.cuda.is_available(), "bench needs a CUDA device"
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    wl = W.WORKLOADS[WORKLOAD]
+    wname, wo_shape = PROFILE_WORKLOADS[args.workload]
+    wl = W.WORKLOADS[wname]
     T, d, k, n = wl.T, wl.d, wl.k, wl.seq_len
-    inp = W.generate_on_device(wl, dev, seed=wl.seed + rank)
+    inp = W.generate_on_device(wl, dev, seed=wl.seed + rank, grad=True)
     u = W.unique_ids(inp["ids_host"])
     g = torch.Generator(device=dev)
     g.manual_seed(wl.seed + 1000 + rank)
-    Wo = (0.02 * torch.randn(*W_O_SHAPE, generator=g, device=dev)).to(torch.bfloat16)
+    Wo = (0.02 * torch.randn(*wo_shape, generator=g, device=dev)).to(torch.bfloat16)
     basis = sn.Basis(inp["U"])
     X, ids, tok, pe, G = inp["X"], inp["ids"], inp["tok_emb"], inp["pos_emb"], inp["G"]
     C = torch.empty(T, k, dtype=torch.bfloat16, device=dev)
@@ -269,7 +285,7 @@ def run_ours(args, world, rank, local, pg):
     Xr = torch.empty_like(X)
     Gr = torch.empty_like(G)
     Wp = torch.empty_like(Wo)
-    ws = torch.empty(max(16, sn.sn_project_weight_workspace(basis, torch.bfloat16, W_O_SHAPE[1])),
+    ws = torch.empty(max(16, sn.sn_project_weight_workspace(basis, torch.bfloat16, wo_shape[1])),
                      dtype=torch.uint8, device=dev)
     wire_f = torch.empty(C.numel() * 2, dtype=torch.uint8, pin_memory=True)
     wire_b = torch.empty(C.numel() * 2, dtype=torch.uint8, pin_memory=True)
@@ -340,7 +356,7 @@ def run_ours(args, world, rank, local, pg):
     value = world * T / (ms / 1e3)
 
     hbm, peak_kind = peaks()
-    ab = algorithmic_bytes(T, d, k, n, u, W_O_SHAPE[1])
+    ab = algorithmic_bytes(T, d, k, n, u, wo_shape[1])
     kernels = {}
     for name in names:
         gbs = ab[name] / (seg[name] / 1e3) / 1e9
@@ -354,44 +370,48 @@ def run_ours(args, world, rank, local, pg):
             traffic = json.load(f).get(dom)
 
     # ---- end to end through the C ABI with host buffers ----
-    Xh = torch.empty(X.shape, dtype=X.dtype, pin_memory=True)
-    Gh = torch.empty(G.shape, dtype=G.dtype, pin_memory=True)
-    idsh = torch.empty(ids.shape, dtype=ids.dtype, pin_memory=True)
-    Xoh = torch.empty_like(Xh, pin_memory=True)
-    Goh = torch.empty_like(Gh, pin_memory=True)
-    Xh.copy_(X)
-    Gh.copy_(G)
-    idsh.copy_(ids)
-    h2d = Xh.numel() * 2 + Gh.numel() * 2 + idsh.numel() * 4
-    d2h = Xoh.numel() * 2 + Goh.numel() * 2
+    e2e_line = None
+    if not args.no_e2e:
+        Xh = torch.empty(X.shape, dtype=X.dtype, pin_memory=True)
+        Gh = torch.empty(G.shape, dtype=G.dtype, pin_memory=True)
+        idsh = torch.empty(ids.shape, dtype=ids.dtype, pin_memory=True)
+        Xoh = torch.empty_like(Xh, pin_memory=True)
+        Goh = torch.empty_like(Gh, pin_memory=True)
+        Xh.copy_(X)
+        Gh.copy_(G)
+        idsh.copy_(ids)
+        h2d = Xh.numel() * 2 + Gh.numel() * 2 + idsh.numel() * 4
+        d2h = Xoh.numel() * 2 + Goh.numel() * 2
 
-    def e2e_step():
-        sn.sn_wire_recv(Xh, X)
-        sn.sn_wire_recv(idsh, ids)
-        sn.sn_wire_recv(Gh, G)
-        step()
-        sn.sn_wire_send(Xr, Xoh)
-        sn.sn_wire_send(Gr, Goh)
+        def e2e_step():
+            sn.sn_wire_recv(Xh, X)
+            sn.sn_wire_recv(idsh, ids)
+            sn.sn_wire_recv(Gh, G)
+            step()
+            sn.sn_wire_send(Xr, Xoh)
+            sn.sn_wire_send(Gr, Goh)
 
-    for _ in range(min(args.warmup, 3)):
-        flush.zero_()
-        e2e_step()
-    torch.cuda.synchronize()
-    e2e_ms = []
-    for _ in range(max(3, args.steps // 2)):
-        flush.zero_()
-        a = torch.cuda.Event(enable_timing=True)
-        b = torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        e2e_step()
-        b.record(stream)
-        b.synchronize()
-        e2e_ms.append(a.elapsed_time(b))
-    sn.sn_check_errors(basis)
-    e2e = max_over_ranks(pg, statistics.mean(e2e_ms), dev)
+        for _ in range(min(args.warmup, 3)):
+            flush.zero_()
+            e2e_step()
+        torch.cuda.synchronize()
+        e2e_ms = []
+        for _ in range(max(3, min(args.steps, 40) // 2)):
+            flush.zero_()
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            e2e_step()
+            b.record(stream)
+            b.synchronize()
+            e2e_ms.append(a.elapsed_time(b))
+        sn.sn_check_errors(basis)
+        e2e = max_over_ranks(pg, statistics.mean(e2e_ms), dev)
+        e2e_line = {"value": world * T / (e2e / 1e3), "unit": "tokens/s",
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e}
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and args.workload == WORKLOAD:
         st, desc, _ = cpu_oracle_step_time(args.cpu_seconds)
         cpu = {"value": T / st, "unit": "tokens/s", "cores": 1, "kind": "oracle",
                "sample": desc}
@@ -401,7 +421,7 @@ def run_ours(args, world, rank, local, pg):
             "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-            "data": "synthetic", "config": config_dict(),
+            "data": "synthetic", "config": config_dict(args.workload),
             "roofline": {"bound": "hbm", "kernel": dom,
                          "achieved": kernels[dom]["gbs"], "peak": hbm,
                          "peak_kind": peak_kind, "unit": "GB/s",
@@ -411,8 +431,7 @@ def run_ours(args, world, rank, local, pg):
             "wire_ms": {"fwd": seg["wire_fwd"], "bwd": seg["wire_bwd"]},
             "boundary_hbm_gbs": sum(ab[nm] for nm in names) / (
                 sum(seg[nm] for nm in names) / 1e3) / 1e9,
-            "e2e": {"value": world * T / (e2e / 1e3), "unit": "tokens/s",
-                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e},
+            "e2e": e2e_line,
             "gpu_launches": launches,
             "unique_ids": u,
             "wall_s_timed_region": wall,

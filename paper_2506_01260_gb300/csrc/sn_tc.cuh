@@ -142,6 +142,10 @@ __device__ __forceinline__ void bulk_wait_read0()
 {
     asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
+__device__ __forceinline__ void bulk_wait_read1()
+{
+    asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+}
 __device__ __forceinline__ void bulk_wait_all0()
 {
     asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");

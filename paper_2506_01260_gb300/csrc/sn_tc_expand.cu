@@ -210,6 +210,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expand(const __grid_constant__ 
         const int tt = threadIdx.x - 64;
         const int row = 32 * q + lane;
         uint32_t g = 0, it = 0;
+        int pend_s = -1;     // stage whose store may still be reading shared memory
         bool ok = true;
         for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++it) {
             const int tile = item / p.chunks, ch = item % p.chunks;
@@ -325,21 +326,41 @@ __global__ void __launch_bounds__(kThreads, 1) k_expand(const __grid_constant__ 
                                           pack_bf16(v[8 * c + 4], v[8 * c + 5]),
                                           pack_bf16(v[8 * c + 6], v[8 * c + 7])));
                 }
+                // Columns past the 8-aligned width of the output map (a TMA store
+                // clips the inner dimension only to 16 bytes) are written directly.
+                const int c0 = blk * BN;
+                if (!GATHER && c0 + BN > p.ncols8 && p.ncols > p.ncols8) {
+                    const int64_t t = r0 + row;
+                    if (t < p.rows) {
+#pragma unroll
+                        for (int e = 0; e < BN; ++e)
+                            if (c0 + e >= p.ncols8 && c0 + e < p.ncols)
+                                p.out[t * p.out_ld + c0 + e] = __float2bfloat16_rn(v[e]);
+                    }
+                }
                 fence_async_smem();
                 __syncwarp();
                 if (lane == 0) {
-                    if (r0 + 32 * q < p.rows) {
-                        tma_store_2d(&p.mapOut, slot + q * 4096, blk * BN, (int)(r0 + 32 * q));
+                    if (r0 + 32 * q < p.rows && c0 < p.ncols8) {
+                        tma_store_2d(&p.mapOut, slot + q * 4096, c0, (int)(r0 + 32 * q));
                         bulk_commit();
-                        bulk_wait_read0();
                     }
-                    mbar_arrive(empty_b + 8 * s);
+                    // release the previous block's stage once its store has read
+                    // shared memory; this block's store stays in flight meanwhile
+                    bulk_wait_read1();
+                    if (pend_s >= 0)
+                        mbar_arrive(empty_b + 8 * pend_s);
                 }
+                pend_s = s;
                 __syncwarp();
             }
         }
-        if (lane == 0)
+        if (lane == 0) {
+            bulk_wait_read0();
+            if (pend_s >= 0)
+                mbar_arrive(empty_b + 8 * pend_s);
             bulk_wait_all0();
+        }
         __syncwarp();
     }
 

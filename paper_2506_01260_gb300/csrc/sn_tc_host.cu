@@ -201,7 +201,7 @@ cudaError_t tc_decompress(const sn_basis &b, const TcArgs &a, __nv_bfloat16 *X_o
     const bool has_pe = a.gather && a.pe != nullptr;
     // the reconstruction stages its output over the (unswizzled) gathered rows
     bool ok = map2d(&p.mapB, b.up16, b.k64, b.d, (uint64_t)b.k64 * 2, 64, BN, true) &&
-              map2d(&p.mapOut, X_out, b.d, a.T, (uint64_t)b.d * 2, 64, 32, !a.gather);
+              map2d(&p.mapOut, X_out, b.d / 8 * 8, a.T, (uint64_t)b.d * 2, 64, 32, !a.gather);
     p.mapA = p.mapB;
     if (ok && a.gather)
         ok = map2d(&p.mapTok, a.tok, b.d, a.vocab, (uint64_t)b.d * 2, 64, 1, false);
@@ -227,7 +227,10 @@ cudaError_t tc_decompress(const sn_basis &b, const TcArgs &a, __nv_bfloat16 *X_o
     p.k = b.k;
     p.katoms = b.k64 / 64;
     p.kmma = b.n_pad / 16;
+    p.out = X_out;
+    p.out_ld = b.d;
     p.ncols = b.d;
+    p.ncols8 = b.d / 8 * 8;
     p.nblk = (b.d + BN - 1) / BN;
     p.ntiles = (int)((a.T + BM - 1) / BM);
     split_blocks(p.ntiles, p.nblk, sms, &p.bpi, &p.chunks);
@@ -291,7 +294,8 @@ cudaError_t tc_project(const sn_basis &b, const __nv_bfloat16 *W, int64_t cols, 
     std::memset(&q, 0, sizeof q);
     ok = map2d(&q.mapA, b.up16, b.k64, b.d, (uint64_t)b.k64 * 2, 64, BM, true) &&
          map2d(&q.mapB, At, b.k64, cols, (uint64_t)b.k64 * 2, 64, BN, true) &&
-         map2d(&q.mapOut, W_out, cols, b.d, (uint64_t)ld * 2, 64, 32, true);
+         map2d(&q.mapOut, W_out, std::max<int64_t>(8, cols / 8 * 8), b.d, (uint64_t)ld * 2, 64,
+               32, true);
     q.mapTok = q.mapPE = q.mapPEg = q.mapB;
     if (!ok)
         return cudaErrorInvalidValue;
@@ -302,7 +306,10 @@ cudaError_t tc_project(const sn_basis &b, const __nv_bfloat16 *W, int64_t cols, 
     q.k = b.k;
     q.katoms = b.k64 / 64;
     q.kmma = b.n_pad / 16;
+    q.out = W_out;
+    q.out_ld = ld;
     q.ncols = (int)cols;
+    q.ncols8 = (int)(cols / 8 * 8);
     q.nblk = (int)((cols + BN - 1) / BN);
     q.ntiles = (b.d + BM - 1) / BM;
     split_blocks(q.ntiles, q.nblk, sms, &q.bpi, &q.chunks);

@@ -76,6 +76,9 @@ struct ExpandParams {
     CUtensorMap mapPE;   // P (SW128, box 64 x 128)
     CUtensorMap mapPEg;  // P (SW128, box 64 x 1, gather4)
     const __nv_bfloat16 *C;   // A by repacking: [rows, k]
+    __nv_bfloat16 *out;       // output base (ragged last columns are stored directly)
+    int64_t out_ld;           // output leading dimension (elements)
+    int ncols8;               // columns covered by mapOut: ncols rounded down to 8
     const int32_t *ids;
     const int32_t *pos;
     unsigned int *err;

@@ -166,12 +166,13 @@ def weight_inputs(cols=None, seed=WEIGHT_SEED, d=WEIGHT_D, k=WEIGHT_K):
 
 # ---- device-side synthesis for full-size workloads -------------------------
 
-def generate_on_device(wl, device, seed=None, dtype="bf16"):
+def generate_on_device(wl, device, seed=None, dtype="bf16", grad=None):
     """Full-size inputs synthesised on the GPU with a seeded torch generator.
 
     Same recipe as `generate`, drawn with torch's device RNG so that gigabyte
     tables never pass through host memory.  U comes from the host fp64 QR.
     Returns torch tensors on `device`; bf16 tensors unless dtype == "f32".
+    `grad` forces (or suppresses) the gradient G regardless of the workload.
     """
     import torch
 
@@ -217,7 +218,7 @@ def generate_on_device(wl, device, seed=None, dtype="bf16"):
         X[t0:t1] = Y.to(tdt)
     del parts
     out = dict(U=U, tok_emb=tok, pos_emb=pe, ids=ids, X=X, ids_host=ids_np)
-    if wl.grad:
+    if wl.grad if grad is None else grad:
         out["G"] = torch.randn(T, d, generator=g, device=device).to(tdt)
     return out
 
