@@ -211,12 +211,13 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16])
 __device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 
 // Instruction descriptor, kind::f16: bf16 A and B (both K-major), fp32 D,
-// shape M x N.
-__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N)
+// shape M x N; `negate_a` computes D (+)= (-A) B.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool negate_a = false)
 {
     return (1u << 4)                     // D format: fp32
            | (1u << 7)                   // A format: bf16
            | (1u << 10)                  // B format: bf16
+           | ((negate_a ? 1u : 0u) << 13)
            | ((uint32_t)(N >> 3) << 17)  // N / 8
            | ((uint32_t)(M >> 4) << 24); // M / 16
 }
@@ -265,6 +266,25 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
     uint32_t r;
     asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
     return r;
+}
+
+// Rewrite a [128 x 128 B] tile of unswizzled rows (as tile::gather4 leaves
+// them) into the 128-byte swizzle layout the MMA reads, in place.  Called by
+// the 128 threads tt = 0..127 of four warps; every row is read and rewritten
+// by one quarter-warp, so only warp-level ordering is needed.
+__device__ __forceinline__ void swizzle_rows_in_place(uint32_t tile, int tt)
+{
+    uint4 v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+        v[u] = lds128(tile + (uint32_t)(tt + 128 * u) * 16);
+    __syncwarp();
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+        const int unit = tt + 128 * u, r = unit >> 3, c = unit & 7;
+        if (r & 7)
+            sts128(tile + sw128(r, c), v[u]);
+    }
 }
 
 __device__ __forceinline__ void named_bar_sync(int id, int nthreads)

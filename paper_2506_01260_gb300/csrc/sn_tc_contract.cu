@@ -11,11 +11,13 @@
 //              gathered rows unswizzled so every gather lands 128-byte aligned);
 //   warp 1     allocates TMEM and issues tcgen05.mma (M = 128, N = k padded
 //              to 16, K = 64 per stage) into a double-buffered fp32 accumulator;
-//   warps 2-5  CMODE_X: subtract the embeddings in fp32 and re-round to bf16
-//              in place (the MMA A operand); CMODE_W: transpose the W tile into
-//              the K-major A operand; then drain the accumulator (tcgen05.ld),
-//              round once to bf16 and store each warp's 32 rows of C as one
-//              contiguous slab.
+//   warps 2-5  CMODE_X: rewrite the gathered rows into the swizzled operand
+//              layout in place; CMODE_W: transpose the W tile into the K-major A
+//              operand; then drain the accumulator (tcgen05.ld), round once to
+//              bf16 and store each warp's 32 rows of C as one contiguous slab.
+// CMODE_X accumulates X U - T_fixed[ids] U - P[pos] U: three MMAs per K-step,
+// the embedding terms with the descriptor's negate-A bit, so the residual is
+// never rounded and the CUDA cores only move bytes.
 // Every wait is bounded; a wait that expires raises SN_EBIT_TIMEOUT and the
 // CTA drains its in-flight copies and MMAs, frees TMEM and returns.
 #include "sn_tc.cuh"
@@ -24,11 +26,6 @@
 namespace sn {
 namespace tc {
 namespace {
-
-__device__ __forceinline__ uint32_t sub3(uint32_t x, uint32_t t, uint32_t p)
-{
-    return pack_bf16(bf_lo(x) - bf_lo(t) - bf_lo(p), bf_hi(x) - bf_hi(t) - bf_hi(p));
-}
 
 template <int MODE>
 __global__ void __launch_bounds__(kThreads, 1) k_contract(const __grid_constant__ ContractParams p)
@@ -156,6 +153,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_contract(const __grid_constant_
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
             const uint32_t idesc = idesc_bf16(BM, p.n_pad);
+            const uint32_t idesc_neg = idesc_bf16(BM, p.n_pad, true);
             uint32_t g = 0, it = 0;
             bool ok = true;
             for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++it) {
@@ -179,11 +177,20 @@ __global__ void __launch_bounds__(kThreads, 1) k_contract(const __grid_constant_
                     }
                     tc_fence_after();
                     const uint32_t st = base + s * pl.stage_bytes;
+                    const uint32_t ub = st + pl.a_bytes;
 #pragma unroll
-                    for (int kk = 0; kk < BK / 16; ++kk)
-                        mma_bf16(d_tmem, sdesc_sw128(st + kk * 32),
-                                 sdesc_sw128(st + pl.a_bytes + kk * 32), idesc,
+                    for (int kk = 0; kk < BK / 16; ++kk) {
+                        const uint64_t bd = sdesc_sw128(ub + kk * 32);
+                        mma_bf16(d_tmem, sdesc_sw128(st + kk * 32), bd, idesc,
                                  (kc > kc0 || kk > 0) ? 1u : 0u);
+                        if (MODE == CMODE_X) {   // - T_fixed[ids] U - P[pos] U
+                            const uint32_t tb = ub + pl.u_bytes;
+                            mma_bf16(d_tmem, sdesc_sw128(tb + kk * 32), bd, idesc_neg, 1u);
+                            if (p.has_pe)
+                                mma_bf16(d_tmem, sdesc_sw128(tb + pl.raw_bytes + kk * 32), bd,
+                                         idesc_neg, 1u);
+                        }
+                    }
                     mma_commit(empty_b + 8 * s);
                 }
                 if (ok)
@@ -208,6 +215,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_contract(const __grid_constant_
             const int kc1 = min(kc0 + p.kc_per_item, kc_total);
             const int64_t r0 = MODE == CMODE_W ? (int64_t)tile * BM
                                                : tile_row0(tile, p.reorder, p.batches, p.seq_len);
+            const bool pe_contig = MODE == CMODE_X && p.has_pe && !p.has_pos &&
+                                   (r0 % p.seq_len) + BM <= p.seq_len;
             if (MODE != CMODE_G) {
                 for (int kc = kc0; kc < kc1; ++kc, ++g) {
                     const int s = g % S;
@@ -218,20 +227,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_contract(const __grid_constant_
                     }
                     const uint32_t st = base + s * pl.stage_bytes;
                     if (MODE == CMODE_X) {
-                        // X tile swizzled; gathered T_fixed / P rows unswizzled (128 B each)
+                        // gathered T_fixed rows (and gathered positional rows) into
+                        // the swizzled layout; a contiguous positional tile arrives
+                        // swizzled already
                         const uint32_t tb = st + pl.a_bytes + pl.u_bytes;
-                        const uint32_t pb = tb + pl.raw_bytes;
-#pragma unroll 4
-                        for (int u = 0; u < 8; ++u) {
-                            const int unit = tt + 128 * u;
-                            const uint32_t xo = sw128(unit >> 3, unit & 7);
-                            const uint32_t po = (uint32_t)unit * 16;
-                            const uint4 x = lds128(st + xo);
-                            const uint4 t = lds128(tb + po);
-                            const uint4 e = p.has_pe ? lds128(pb + po) : make_uint4(0, 0, 0, 0);
-                            sts128(st + xo, make_uint4(sub3(x.x, t.x, e.x), sub3(x.y, t.y, e.y),
-                                                       sub3(x.z, t.z, e.z), sub3(x.w, t.w, e.w)));
-                        }
+                        swizzle_rows_in_place(tb, tt);
+                        if (p.has_pe && !pe_contig)
+                            swizzle_rows_in_place(tb + pl.raw_bytes, tt);
                     } else {   // CMODE_W: raw W tile [64 d][128 c] -> A operand [128 c][64 d]
                         const uint32_t raw = st + pl.a_bytes + pl.u_bytes;
 #pragma unroll

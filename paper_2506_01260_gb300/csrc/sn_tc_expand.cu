@@ -7,16 +7,20 @@
 // A work item is one 128-row tile and a run of 64-column output blocks.
 //   warp 0     TMA producer: per block, the 64 rows of the B operand (U, or
 //              A^T; 128-byte swizzled) and, for the reconstruction, the gathered
-//              T_fixed rows (tile::gather4) and positional rows (unswizzled);
-//              per item, the A operand rows when they come from a tensor map;
-//   warp 1     TMEM allocation and tcgen05.mma (M = 128, N = 64, K = k padded
-//              to 16) into a double-buffered fp32 accumulator;
+//              T_fixed rows (tile::gather4, unswizzled) and the positional rows
+//              (one swizzled tile when the positions are contiguous, else
+//              gathered); per item, the A operand when it comes from a tensor map;
+//   warp 1     TMEM allocation and tcgen05.mma into a double-buffered fp32
+//              accumulator (M = 128, N = 64): C U^T over K = k padded to 16,
+//              then, for the reconstruction, + T_fixed rows . I + P rows . I
+//              with a resident 64 x 64 identity operand, so the embeddings are
+//              added in fp32 inside the tensor core;
 //   warps 2-5  per item, repack the item's C rows into the swizzled K-major A
-//              operand (zero-padded to the MMA K); per block, drain the
-//              accumulator, add the positional and token rows in fp32, round
-//              once to bf16 into shared memory (over the gathered rows), and
-//              TMA-store each warp's 32 rows (rows past the end are clipped by
-//              the tensor map).
+//              operand (zero-padded); per block, drain the accumulator, round
+//              once to bf16 into a swizzled staging tile and TMA-store each
+//              warp's 32 rows (rows past the end are clipped by the map);
+//   warps 6-9  (reconstruction only) build the identity, then rewrite each
+//              block's gathered rows into the swizzled operand layout.
 // Every wait is bounded (SN_EBIT_TIMEOUT); an aborting CTA drains its copies
 // and MMAs and frees TMEM before it returns.
 #include "sn_tc.cuh"
@@ -26,13 +30,9 @@ namespace sn {
 namespace tc {
 namespace {
 
-__device__ __forceinline__ uint32_t add3(float a0, float a1, uint32_t p, uint32_t t)
-{
-    return pack_bf16(a0 + bf_lo(p) + bf_lo(t), a1 + bf_hi(p) + bf_hi(t));
-}
-
 template <int AMODE, bool GATHER>
-__global__ void __launch_bounds__(kThreads, 1) k_expand(const __grid_constant__ ExpandParams p)
+__global__ void __launch_bounds__(expand_threads(GATHER), 1)
+    k_expand(const __grid_constant__ ExpandParams p)
 {
     extern __shared__ uint8_t smem_raw[];
     uint32_t base = smem_u32(smem_raw);
@@ -42,12 +42,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_expand(const __grid_constant__ 
 
     const int S = p.stages;
     const ExpandPlan pl = expand_plan(GATHER, p.katoms, p.has_pe, S);
-    const uint32_t a_s = base;
+    const uint32_t a_s = base, id_s = base + pl.a_bytes;
+    const uint32_t stage0 = base + pl.a_bytes + pl.id_bytes;
     const uint32_t bar = base + pl.bar_off;
-    const uint32_t full_b = bar, empty_b = bar + 8 * S;
-    const uint32_t accf_b = bar + 16 * S, acce_b = accf_b + 16;
+    const uint32_t full_b = bar, empty_b = bar + 8 * S, tready_b = bar + 16 * S;
+    const uint32_t accf_b = bar + 24 * S, acce_b = accf_b + 16;
     const uint32_t afull_b = acce_b + 16, aempty_b = afull_b + 8, drain_b = aempty_b + 8;
-    uint32_t *tmem_slot = (uint32_t *)(smem + pl.bar_off + 8 * (2 * S + 7));
+    const uint32_t idready_b = drain_b + 8;
+    uint32_t *tmem_slot = (uint32_t *)(smem + pl.bar_off + 8 * (3 * S + 8));
     volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     constexpr uint32_t kTmemCols = 2 * BN;
@@ -56,6 +58,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expand(const __grid_constant__ 
         for (int s = 0; s < S; ++s) {
             mbar_init(full_b + 8 * s, 1);
             mbar_init(empty_b + 8 * s, 4);
+            mbar_init(tready_b + 8 * s, 4);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(accf_b + 8 * b, 1);
@@ -64,6 +67,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expand(const __grid_constant__ 
         mbar_init(afull_b, AMODE == AMODE_REPACK ? 4 : 1);
         mbar_init(aempty_b, 1);
         mbar_init(drain_b, 1);
+        mbar_init(idready_b, 4);
         *abort_flag = 0;
         mbar_fence_init();
     }
@@ -136,7 +140,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expand(const __grid_constant__ 
                     ok = false;
                     break;
                 }
-                const uint32_t st = base + pl.a_bytes + s * pl.stage_bytes;
+                const uint32_t st = stage0 + s * pl.stage_bytes;
                 const uint32_t fb = full_b + 8 * s;
                 if (lane == 0)
                     mbar_arrive_tx(fb, pl.tx_bytes);
@@ -170,6 +174,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_expand(const __grid_constant__ 
             const uint32_t idesc = idesc_bf16(BM, BN);
             uint32_t g = 0, it = 0;
             bool ok = true;
+            if (GATHER && !mbar_wait(idready_b, 0, abort_flag, p.err))
+                ok = false;
             for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++it) {
                 const int ch = item % p.chunks;
                 const int blk0 = ch * p.bpi, blk1 = min(blk0 + p.bpi, p.nblk);
@@ -187,11 +193,28 @@ __global__ void __launch_bounds__(kThreads, 1) k_expand(const __grid_constant__ 
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t st = base + pl.a_bytes + s * pl.stage_bytes;
+                    const uint32_t st = stage0 + s * pl.stage_bytes;
+                    const uint32_t d_tmem = tmem + b * BN;
                     for (int kk = 0; kk < p.kmma; ++kk) {
                         const uint32_t a = kk >> 2, off = (kk & 3) * 32;
-                        mma_bf16(tmem + b * BN, sdesc_sw128(a_s + a * kTile + off),
+                        mma_bf16(d_tmem, sdesc_sw128(a_s + a * kTile + off),
                                  sdesc_sw128(st + a * (BN * 128) + off), idesc, kk > 0 ? 1u : 0u);
+                    }
+                    if (GATHER) {   // + T_fixed rows . I + P rows . I
+                        if (!mbar_wait(tready_b + 8 * s, n & 1, abort_flag, p.err)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t tb = st + pl.b_bytes;
+#pragma unroll
+                        for (int kk = 0; kk < BN / 16; ++kk) {
+                            const uint64_t idd = sdesc_sw128(id_s + kk * 32);
+                            mma_bf16(d_tmem, sdesc_sw128(tb + kk * 32), idd, idesc, 1u);
+                            if (p.has_pe)
+                                mma_bf16(d_tmem, sdesc_sw128(tb + kTile + kk * 32), idd, idesc,
+                                         1u);
+                        }
                     }
                     mma_commit(accf_b + 8 * b);
                 }
@@ -204,8 +227,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_expand(const __grid_constant__ 
             }
         }
         __syncwarp();
-    } else {
-        // ------------------------------------------------------------ compute warps
+    } else if (warp < 6) {
+        // ------------------------------------------------------------ epilogue warps
         const int q = warp & 3;
         const int tt = threadIdx.x - 64;
         const int row = 32 * q + lane;
@@ -264,7 +287,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_expand(const __grid_constant__ 
             }
             for (int blk = blk0; blk < blk1; ++blk, ++g) {
                 const int s = g % S;
-                const uint32_t n = g / S, b = g & 1, nb = g >> 1;
+                const uint32_t b = g & 1, nb = g >> 1;
                 if (!warp_wait(accf_b + 8 * b, nb & 1, abort_flag, p.err)) {
                     ok = false;
                     break;
@@ -280,51 +303,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_expand(const __grid_constant__ 
                 __syncwarp();
                 if (lane == 0)
                     mbar_arrive(acce_b + 8 * b);
-                if (GATHER && !warp_wait(full_b + 8 * s, n & 1, abort_flag, p.err)) {
-                    ok = false;
-                    break;
-                }
-                const uint32_t slot = base + pl.a_bytes + s * pl.stage_bytes + pl.b_bytes;
-                const uint32_t pslot = slot + kTile;
-                if (GATHER) {
-                    // Gathered rows are unswizzled 128-byte rows, so a thread (one row)
-                    // walks its 16-byte chunks starting at chunk (row & 7): the 8 rows of
-                    // a quarter-warp then touch 8 different banks.  Rotate the
-                    // accumulator by the same amount so chunk c of v is chunk
-                    // (c + rot) & 7 of the row.
-                    const int rot = row & 7;
+                // the output tile is staged over the block's T_fixed rows, which
+                // the MMA has finished reading
+                const uint32_t slot = stage0 + s * pl.stage_bytes + pl.b_bytes;
 #pragma unroll
-                    for (int sh = 1; sh <= 4; sh <<= 1) {
-                        const bool on = (rot & sh) != 0;
-                        float w[BN];
-#pragma unroll
-                        for (int i = 0; i < BN; ++i)
-                            w[i] = on ? v[(i + 8 * sh) & (BN - 1)] : v[i];
-#pragma unroll
-                        for (int i = 0; i < BN; ++i)
-                            v[i] = w[i];
-                    }
-#pragma unroll
-                    for (int c = 0; c < 8; ++c) {
-                        const uint32_t off = (uint32_t)row * 128 + (((c + rot) & 7) << 4);
-                        const uint4 tv = lds128(slot + off);
-                        const uint4 pv = p.has_pe ? lds128(pslot + off) : make_uint4(0, 0, 0, 0);
-                        uint4 o = make_uint4(add3(v[8 * c + 0], v[8 * c + 1], pv.x, tv.x),
-                                             add3(v[8 * c + 2], v[8 * c + 3], pv.y, tv.y),
-                                             add3(v[8 * c + 4], v[8 * c + 5], pv.z, tv.z),
-                                             add3(v[8 * c + 6], v[8 * c + 7], pv.w, tv.w));
-                        if (bad)
-                            o = make_uint4(0, 0, 0, 0);
-                        sts128(slot + off, o);       // in place: the store map is unswizzled
-                    }
-                } else {
-#pragma unroll
-                    for (int c = 0; c < 8; ++c)      // swizzled staging, swizzled store map
-                        sts128(slot + sw128(row, c),
-                               make_uint4(pack_bf16(v[8 * c + 0], v[8 * c + 1]),
-                                          pack_bf16(v[8 * c + 2], v[8 * c + 3]),
-                                          pack_bf16(v[8 * c + 4], v[8 * c + 5]),
-                                          pack_bf16(v[8 * c + 6], v[8 * c + 7])));
+                for (int c = 0; c < 8; ++c) {
+                    uint4 o = make_uint4(pack_bf16(v[8 * c + 0], v[8 * c + 1]),
+                                         pack_bf16(v[8 * c + 2], v[8 * c + 3]),
+                                         pack_bf16(v[8 * c + 4], v[8 * c + 5]),
+                                         pack_bf16(v[8 * c + 6], v[8 * c + 7]));
+                    if (bad)
+                        o = make_uint4(0, 0, 0, 0);
+                    sts128(slot + sw128(row, c), o);
                 }
                 // Columns past the 8-aligned width of the output map (a TMA store
                 // clips the inner dimension only to 16 bytes) are written directly.
@@ -362,6 +352,47 @@ __global__ void __launch_bounds__(kThreads, 1) k_expand(const __grid_constant__ 
             bulk_wait_all0();
         }
         __syncwarp();
+    } else if (GATHER) {
+        // ------------------------------------------------------------ row-layout warps
+        const int tt = threadIdx.x - 192;    // 0..127
+        // identity B operand: 64 rows (N) x 64 columns (K), swizzled
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int unit = tt + 128 * u, n = unit >> 3, c = unit & 7;
+            // row n holds bf16 1.0 at column n: chunk n / 8, element n % 8
+            const uint32_t one = (n & 1) ? 0x3F800000u : 0x00003F80u;
+            const int word = ((n >> 3) == c) ? ((n & 7) >> 1) : -1;
+            sts128(id_s + sw128(n, c), make_uint4(word == 0 ? one : 0u, word == 1 ? one : 0u,
+                                                  word == 2 ? one : 0u, word == 3 ? one : 0u));
+        }
+        fence_async_smem();
+        __syncwarp();
+        if (lane == 0)
+            mbar_arrive(idready_b);
+        uint32_t g = 0;
+        bool ok = true;
+        for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x) {
+            const int tile = item / p.chunks, ch = item % p.chunks;
+            const int blk0 = ch * p.bpi, blk1 = min(blk0 + p.bpi, p.nblk);
+            const int64_t r0 = tile_row0(tile, p.reorder, p.batches, p.seq_len);
+            const bool pe_contig = p.has_pe && !p.has_pos && (r0 % p.seq_len) + BM <= p.seq_len;
+            for (int blk = blk0; blk < blk1; ++blk, ++g) {
+                const int s = g % S;
+                const uint32_t n = g / S;
+                if (!warp_wait(full_b + 8 * s, n & 1, abort_flag, p.err)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t tb = stage0 + s * pl.stage_bytes + pl.b_bytes;
+                swizzle_rows_in_place(tb, tt);
+                if (p.has_pe && !pe_contig)
+                    swizzle_rows_in_place(tb + kTile, tt);
+                fence_async_smem();
+                __syncwarp();
+                if (lane == 0)
+                    mbar_arrive(tready_b + 8 * s);
+            }
+        }
     }
 
     tc_fence_before();
@@ -377,22 +408,23 @@ __global__ void __launch_bounds__(kThreads, 1) k_expand(const __grid_constant__ 
 cudaError_t launch_expand(int amode, bool gather, const ExpandParams &p, int grid, cudaStream_t s)
 {
     const ExpandPlan pl = expand_plan(gather, p.katoms, p.has_pe, p.stages);
+    const int threads = expand_threads(gather);
     cudaError_t e;
     if (amode == AMODE_REPACK && gather) {
         e = cudaFuncSetAttribute(k_expand<AMODE_REPACK, true>,
                                  cudaFuncAttributeMaxDynamicSharedMemorySize, pl.total);
         if (e == cudaSuccess)
-            k_expand<AMODE_REPACK, true><<<grid, kThreads, pl.total, s>>>(p);
+            k_expand<AMODE_REPACK, true><<<grid, threads, pl.total, s>>>(p);
     } else if (amode == AMODE_REPACK) {
         e = cudaFuncSetAttribute(k_expand<AMODE_REPACK, false>,
                                  cudaFuncAttributeMaxDynamicSharedMemorySize, pl.total);
         if (e == cudaSuccess)
-            k_expand<AMODE_REPACK, false><<<grid, kThreads, pl.total, s>>>(p);
+            k_expand<AMODE_REPACK, false><<<grid, threads, pl.total, s>>>(p);
     } else {
         e = cudaFuncSetAttribute(k_expand<AMODE_TMA, false>,
                                  cudaFuncAttributeMaxDynamicSharedMemorySize, pl.total);
         if (e == cudaSuccess)
-            k_expand<AMODE_TMA, false><<<grid, kThreads, pl.total, s>>>(p);
+            k_expand<AMODE_TMA, false><<<grid, threads, pl.total, s>>>(p);
     }
     if (e != cudaSuccess)
         return e;

@@ -162,7 +162,7 @@ cudaError_t tc_compress(const sn_basis &b, const TcArgs &a, cudaStream_t s)
     else
         p.mapTok = p.mapA;
     if (ok && has_pe)
-        ok = map2d(&p.mapPE, a.pe, b.d, a.seq_len, (uint64_t)b.d * 2, BK, BM, false) &&
+        ok = map2d(&p.mapPE, a.pe, b.d, a.seq_len, (uint64_t)b.d * 2, BK, BM, true) &&
              map2d(&p.mapPEg, a.pe, b.d, a.seq_len, (uint64_t)b.d * 2, BK, 1, false);
     else
         p.mapPE = p.mapPEg = p.mapA;
@@ -199,16 +199,17 @@ cudaError_t tc_decompress(const sn_basis &b, const TcArgs &a, __nv_bfloat16 *X_o
     ExpandParams p;
     std::memset(&p, 0, sizeof p);
     const bool has_pe = a.gather && a.pe != nullptr;
-    // the reconstruction stages its output over the (unswizzled) gathered rows
+    // gathered rows land unswizzled (every tile::gather4 destination is then
+    // 128-byte aligned) and are rewritten in shared memory; tiles are swizzled
     bool ok = map2d(&p.mapB, b.up16, b.k64, b.d, (uint64_t)b.k64 * 2, 64, BN, true) &&
-              map2d(&p.mapOut, X_out, b.d / 8 * 8, a.T, (uint64_t)b.d * 2, 64, 32, !a.gather);
+              map2d(&p.mapOut, X_out, b.d / 8 * 8, a.T, (uint64_t)b.d * 2, 64, 32, true);
     p.mapA = p.mapB;
     if (ok && a.gather)
         ok = map2d(&p.mapTok, a.tok, b.d, a.vocab, (uint64_t)b.d * 2, 64, 1, false);
     else
         p.mapTok = p.mapB;
     if (ok && has_pe)
-        ok = map2d(&p.mapPE, a.pe, b.d, a.seq_len, (uint64_t)b.d * 2, 64, BM, false) &&
+        ok = map2d(&p.mapPE, a.pe, b.d, a.seq_len, (uint64_t)b.d * 2, 64, BM, true) &&
              map2d(&p.mapPEg, a.pe, b.d, a.seq_len, (uint64_t)b.d * 2, 64, 1, false);
     else
         p.mapPE = p.mapPEg = p.mapB;

@@ -23,9 +23,9 @@ enum { CMODE_G = 0, CMODE_X = 1, CMODE_W = 2 };
 struct ContractParams {
     CUtensorMap mapA;    // X or G [T, d] (SW128, box 64 x 128) | W [d, m] (plain, box 128 x 64)
     CUtensorMap mapU;    // U^T padded [n_pad, d] (SW128, box 64 x n_pad)
-    CUtensorMap mapTok;  // T_fixed [vocab, d] (SW128, box 64 x 1, gather4)
+    CUtensorMap mapTok;  // T_fixed [vocab, d] (plain, box 64 x 1, gather4)
     CUtensorMap mapPE;   // P [seq_len, d] (SW128, box 64 x 128)
-    CUtensorMap mapPEg;  // P [seq_len, d] (SW128, box 64 x 1, gather4)
+    CUtensorMap mapPEg;  // P [seq_len, d] (plain, box 64 x 1, gather4)
     const int32_t *ids;
     const int32_t *pos;
     __nv_bfloat16 *C;    // [T, k] output (G, X modes)
@@ -72,9 +72,9 @@ struct ExpandParams {
     CUtensorMap mapA;    // A by TMA: U padded [d, k64] (SW128, box 64 x 128)
     CUtensorMap mapB;    // B rows: U padded [d, k64] | A^T [m, k64] (SW128, box 64 x 64)
     CUtensorMap mapOut;  // output [rows, ncols] (SW128, box 64 x 32)
-    CUtensorMap mapTok;  // T_fixed (SW128, box 64 x 1, gather4)
+    CUtensorMap mapTok;  // T_fixed (plain, box 64 x 1, gather4)
     CUtensorMap mapPE;   // P (SW128, box 64 x 128)
-    CUtensorMap mapPEg;  // P (SW128, box 64 x 1, gather4)
+    CUtensorMap mapPEg;  // P (plain, box 64 x 1, gather4)
     const __nv_bfloat16 *C;   // A by repacking: [rows, k]
     __nv_bfloat16 *out;       // output base (ragged last columns are stored directly)
     int64_t out_ld;           // output leading dimension (elements)
@@ -92,23 +92,29 @@ struct ExpandParams {
 };
 
 struct ExpandPlan {
-    uint32_t a_bytes, b_bytes, out_bytes, pe_bytes, stage_bytes, bar_off, total, tx_bytes;
+    uint32_t a_bytes, id_bytes, b_bytes, out_bytes, pe_bytes, stage_bytes, bar_off, total,
+        tx_bytes;
 };
 
+// Shared memory of the expansion: A operand | identity (gather) | stages of
+// [B rows | T_fixed rows, later the output tile | positional rows] | barriers.
 __host__ __device__ inline ExpandPlan expand_plan(bool gather, int katoms, int has_pe,
                                                   int stages)
 {
     ExpandPlan p;
     p.a_bytes = (uint32_t)katoms * kTile;
+    p.id_bytes = gather ? BN * 128 : 0;           // 64 x 64 bf16 identity, swizzled
     p.b_bytes = (uint32_t)katoms * BN * 128;
-    p.out_bytes = kTile;                           // T_fixed rows, overwritten by the output
+    p.out_bytes = kTile;
     p.pe_bytes = (gather && has_pe) ? kTile : 0;
     p.stage_bytes = p.b_bytes + p.out_bytes + p.pe_bytes;
-    p.bar_off = p.a_bytes + (uint32_t)stages * p.stage_bytes;
-    p.total = p.bar_off + 8 * (2 * stages + 7) + 16 + 1024;
+    p.bar_off = p.a_bytes + p.id_bytes + (uint32_t)stages * p.stage_bytes;
+    p.total = p.bar_off + 8 * (3 * stages + 8) + 16 + 1024;
     p.tx_bytes = p.b_bytes + (gather ? p.out_bytes + p.pe_bytes : 0);
     return p;
 }
+
+__host__ __device__ constexpr int expand_threads(bool gather) { return gather ? 320 : 192; }
 
 // Row tile -> first row.  With `reorder`, tiles run position-block-major so the
 // b sequences of a batch that share positional rows are processed together
