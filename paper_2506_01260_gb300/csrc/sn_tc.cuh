@@ -268,6 +268,40 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
     return r;
 }
 
+// ---- cp.async: 16-byte global -> shared copies issued per thread -------------
+// Used for row gathers: each thread places its chunks directly at their
+// swizzled positions.  Completion is observed with wait_group by the issuing
+// thread, which then fences toward the async proxy before arriving on the
+// stage's mbarrier.
+// Copies `src_bytes` (0 or 16) bytes and zero-fills the rest of the 16.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, uint32_t src_bytes)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
+                 "r"(src_bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait0() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+
+// Row gather of one [128 x 64] bf16 tile: thread tt (0..127) copies chunk
+// (tt & 7) of rows (tt >> 3) + 16 u, u = 0..7, from src_rows[u] (element
+// offsets into `table`) + col0, into the swizzled tile at `dst`.  Columns at
+// or past `row_len` (a ragged last chunk) are zero-filled without a read.
+__device__ __forceinline__ void gather_tile_async(uint32_t dst, const __nv_bfloat16 *table,
+                                                  const int64_t (&src_rows)[8], int64_t col0,
+                                                  int64_t row_len, int tt)
+{
+    const int c = tt & 7;
+    const int64_t col = col0 + 8 * c;
+    const bool in = col + 8 <= row_len;       // row_len is a multiple of 8
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+        const int r = (tt >> 3) + 16 * u;
+        cp_async16(dst + sw128(r, c), table + src_rows[u] + (in ? col : 0), in ? 16u : 0u);
+    }
+}
+
 // Rewrite a [128 x 128 B] tile of unswizzled rows (as tile::gather4 leaves
 // them) into the 128-byte swizzle layout the MMA reads, in place.  Called by
 // the 128 threads tt = 0..127 of four warps; every row is read and rewritten

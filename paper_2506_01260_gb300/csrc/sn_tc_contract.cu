@@ -4,20 +4,22 @@
 //   CMODE_G  C[t, :] = G[t, :] U                                       Sec. 4.4, Eq. (grad_compress)
 //   CMODE_W  A^T[c, :] = W[:, c]^T U  (fp32 partials over a d-range)    first pass of W' = U (U^T W)
 //
-// Persistent CTAs of six warps walk 128-row tiles:
-//   warp 0     TMA producer: the X/G tile, the U^T chunk, and (CMODE_X) the
-//              gathered T_fixed rows (tile::gather4) and positional rows into
-//              a ring of shared-memory stages (X and U^T 128-byte swizzled,
-//              gathered rows unswizzled so every gather lands 128-byte aligned);
+// Persistent CTAs walk 128-row tiles in 64-column chunks of d through a ring
+// of shared-memory stages (all operand tiles 128-byte swizzled, K-major):
+//   warp 0     TMA producer: the X/G tile (or raw W tile), the U^T chunk and,
+//              when a tile's positions are contiguous, the positional tile;
 //   warp 1     allocates TMEM and issues tcgen05.mma (M = 128, N = k padded
-//              to 16, K = 64 per stage) into a double-buffered fp32 accumulator;
-//   warps 2-5  CMODE_X: rewrite the gathered rows into the swizzled operand
-//              layout in place; CMODE_W: transpose the W tile into the K-major A
-//              operand; then drain the accumulator (tcgen05.ld), round once to
-//              bf16 and store each warp's 32 rows of C as one contiguous slab.
-// CMODE_X accumulates X U - T_fixed[ids] U - P[pos] U: three MMAs per K-step,
-// the embedding terms with the descriptor's negate-A bit, so the residual is
-// never rounded and the CUDA cores only move bytes.
+//              to 16, K = 16) into a double-buffered fp32 accumulator.  CMODE_X
+//              accumulates X U - T_fixed[ids] U - P[pos] U: three MMAs per
+//              K-step, the embedding terms with the descriptor's negate-A bit,
+//              so the residual is never rounded;
+//   warps 2-5  CMODE_W: transpose the raw W tile into the K-major A operand;
+//              then drain the accumulator (tcgen05.ld), round once to bf16 and
+//              store each warp's 32 rows of C as one contiguous slab (CMODE_W:
+//              fp32 partial rows);
+//   warps 6-9  CMODE_X: gather the T_fixed rows (and non-contiguous positional
+//              rows) with 16-byte cp.async copies straight into their swizzled
+//              positions, then fence toward the async proxy and arrive.
 // Every wait is bounded; a wait that expires raises SN_EBIT_TIMEOUT and the
 // CTA drains its in-flight copies and MMAs, frees TMEM and returns.
 #include "sn_tc.cuh"
@@ -28,7 +30,8 @@ namespace tc {
 namespace {
 
 template <int MODE>
-__global__ void __launch_bounds__(kThreads, 1) k_contract(const __grid_constant__ ContractParams p)
+__global__ void __launch_bounds__(contract_threads(MODE), 1)
+    k_contract(const __grid_constant__ ContractParams p)
 {
     extern __shared__ uint8_t smem_raw[];
     uint32_t base = smem_u32(smem_raw);
@@ -48,7 +51,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_contract(const __grid_constant_
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
-            mbar_init(full_b + 8 * s, 1);
+            mbar_init(full_b + 8 * s, MODE == CMODE_X ? 1 + 4 : 1);
             mbar_init(rr_b + 8 * s, 4);
             mbar_init(empty_b + 8 * s, 1);
         }
@@ -71,17 +74,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_contract(const __grid_constant_
     const int kc_total = p.nkc;
 
     if (warp == 0) {
-        // ------------------------------------------------------------ producer
+        // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
             tma_prefetch(&p.mapA);
             tma_prefetch(&p.mapU);
-            if (MODE == CMODE_X) {
-                tma_prefetch(&p.mapTok);
-                if (p.has_pe) {
-                    tma_prefetch(&p.mapPE);
-                    tma_prefetch(&p.mapPEg);
-                }
-            }
+            if (MODE == CMODE_X && p.has_pe)
+                tma_prefetch(&p.mapPE);
         }
         uint32_t g = 0;
         bool ok = true;
@@ -91,28 +89,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_contract(const __grid_constant_
             const int kc1 = min(kc0 + p.kc_per_item, kc_total);
             const int64_t r0 = MODE == CMODE_W ? (int64_t)tile * BM
                                                : tile_row0(tile, p.reorder, p.batches, p.seq_len);
-            int rid[4] = {0, 0, 0, 0}, rps[4] = {0, 0, 0, 0};
-            bool pe_tile = false;
-            if (MODE == CMODE_X) {
-#pragma unroll
-                for (int r = 0; r < 4; ++r) {
-                    const int64_t t = r0 + 4 * lane + r;
-                    int id = 0, ps = 0;
-                    if (t < p.rows) {
-                        id = p.ids[t];
-                        if (id < 0 || id >= p.vocab)
-                            id = 0;                       // row zeroed by the epilogue
-                        if (p.has_pe) {
-                            ps = p.has_pos ? p.pos[t] : (int)(t % p.seq_len);
-                            if (ps < 0 || ps >= p.seq_len)
-                                ps = 0;
-                        }
-                    }
-                    rid[r] = id;
-                    rps[r] = ps;
-                }
-                pe_tile = p.has_pe && !p.has_pos && (r0 % p.seq_len) + BM <= p.seq_len;
-            }
+            const bool pe_tile = MODE == CMODE_X && p.has_pe && !p.has_pos &&
+                                 (r0 % p.seq_len) + BM <= p.seq_len;
+            const uint32_t tx = MODE == CMODE_W ? pl.raw_bytes + pl.u_bytes
+                                                : pl.a_bytes + pl.u_bytes + (pe_tile ? kTile : 0);
             for (int kc = kc0; kc < kc1; ++kc, ++g) {
                 const int s = g % S;
                 const uint32_t n = g / S;
@@ -122,26 +102,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_contract(const __grid_constant_
                 }
                 const uint32_t st = base + s * pl.stage_bytes;
                 const uint32_t fb = full_b + 8 * s;
-                if (lane == 0)
-                    mbar_arrive_tx(fb, pl.tx_bytes);
-                __syncwarp();
                 if (lane == 0) {
+                    mbar_arrive_tx(fb, tx);
                     if (MODE == CMODE_W)
                         tma_load_2d(st + pl.a_bytes + pl.u_bytes, &p.mapA, (int)r0, kc * BK, fb);
                     else
                         tma_load_2d(st, &p.mapA, kc * BK, (int)r0, fb);
                     tma_load_2d(st + pl.a_bytes, &p.mapU, kc * BK, 0, fb);
-                    if (MODE == CMODE_X && pe_tile)
+                    if (pe_tile)
                         tma_load_2d(st + pl.a_bytes + pl.u_bytes + pl.raw_bytes, &p.mapPE,
                                     kc * BK, (int)(r0 % p.seq_len), fb);
                 }
-                if (MODE == CMODE_X) {
-                    tma_gather4(st + pl.a_bytes + pl.u_bytes + lane * 512, &p.mapTok, kc * BK,
-                                rid[0], rid[1], rid[2], rid[3], fb);
-                    if (p.has_pe && !pe_tile)
-                        tma_gather4(st + pl.a_bytes + pl.u_bytes + pl.raw_bytes + lane * 512,
-                                    &p.mapPEg, kc * BK, rps[0], rps[1], rps[2], rps[3], fb);
-                }
+                __syncwarp();
             }
         }
         if (!ok && lane == 0) {   // let copies already issued land before the CTA exits
@@ -170,7 +142,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_contract(const __grid_constant_
                 for (int kc = kc0; kc < kc1; ++kc, ++g) {
                     const int s = g % S;
                     const uint32_t n = g / S;
-                    const uint32_t wb = (MODE == CMODE_G ? full_b : rr_b) + 8 * s;
+                    const uint32_t wb = (MODE == CMODE_W ? rr_b : full_b) + 8 * s;
                     if (!mbar_wait(wb, n & 1, abort_flag, p.err)) {
                         ok = false;
                         break;
@@ -202,8 +174,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_contract(const __grid_constant_
             }
         }
         __syncwarp();
-    } else {
-        // ------------------------------------------------------------ compute warps
+    } else if (warp < 6) {
+        // ------------------------------------------------------------ epilogue warps
         const int q = warp & 3;              // TMEM lane quarter of this warp
         const int tt = threadIdx.x - 64;     // 0..127
         const int row = 32 * q + lane;
@@ -215,9 +187,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_contract(const __grid_constant_
             const int kc1 = min(kc0 + p.kc_per_item, kc_total);
             const int64_t r0 = MODE == CMODE_W ? (int64_t)tile * BM
                                                : tile_row0(tile, p.reorder, p.batches, p.seq_len);
-            const bool pe_contig = MODE == CMODE_X && p.has_pe && !p.has_pos &&
-                                   (r0 % p.seq_len) + BM <= p.seq_len;
-            if (MODE != CMODE_G) {
+            if (MODE == CMODE_W) {
                 for (int kc = kc0; kc < kc1; ++kc, ++g) {
                     const int s = g % S;
                     const uint32_t n = g / S;
@@ -225,33 +195,24 @@ __global__ void __launch_bounds__(kThreads, 1) k_contract(const __grid_constant_
                         ok = false;
                         break;
                     }
+                    // raw W tile [64 d][128 c] -> A operand [128 c][64 d]
                     const uint32_t st = base + s * pl.stage_bytes;
-                    if (MODE == CMODE_X) {
-                        // gathered T_fixed rows (and gathered positional rows) into
-                        // the swizzled layout; a contiguous positional tile arrives
-                        // swizzled already
-                        const uint32_t tb = st + pl.a_bytes + pl.u_bytes;
-                        swizzle_rows_in_place(tb, tt);
-                        if (p.has_pe && !pe_contig)
-                            swizzle_rows_in_place(tb + pl.raw_bytes, tt);
-                    } else {   // CMODE_W: raw W tile [64 d][128 c] -> A operand [128 c][64 d]
-                        const uint32_t raw = st + pl.a_bytes + pl.u_bytes;
+                    const uint32_t raw = st + pl.a_bytes + pl.u_bytes;
 #pragma unroll
-                        for (int c = 0; c < 8; ++c) {
-                            uint32_t w[4];
+                    for (int c = 0; c < 8; ++c) {
+                        uint32_t w[4];
 #pragma unroll
-                            for (int e = 0; e < 4; ++e) {
-                                unsigned short lo, hi;
-                                asm volatile("ld.shared.u16 %0, [%1];"
-                                             : "=h"(lo)
-                                             : "r"(raw + (8 * c + 2 * e) * 256 + tt * 2));
-                                asm volatile("ld.shared.u16 %0, [%1];"
-                                             : "=h"(hi)
-                                             : "r"(raw + (8 * c + 2 * e + 1) * 256 + tt * 2));
-                                w[e] = (uint32_t)lo | ((uint32_t)hi << 16);
-                            }
-                            sts128(st + sw128(tt, c), make_uint4(w[0], w[1], w[2], w[3]));
+                        for (int e = 0; e < 4; ++e) {
+                            unsigned short lo, hi;
+                            asm volatile("ld.shared.u16 %0, [%1];"
+                                         : "=h"(lo)
+                                         : "r"(raw + (8 * c + 2 * e) * 256 + tt * 2));
+                            asm volatile("ld.shared.u16 %0, [%1];"
+                                         : "=h"(hi)
+                                         : "r"(raw + (8 * c + 2 * e + 1) * 256 + tt * 2));
+                            w[e] = (uint32_t)lo | ((uint32_t)hi << 16);
                         }
+                        sts128(st + sw128(tt, c), make_uint4(w[0], w[1], w[2], w[3]));
                     }
                     fence_async_smem();
                     __syncwarp();
@@ -261,7 +222,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_contract(const __grid_constant_
                 if (!ok)
                     break;
             }
-            // ---- epilogue: accumulator -> output
+            // ---- accumulator -> output
             const uint32_t b = it & 1, nb = it >> 1;
             if (!warp_wait(accf_b + 8 * b, nb & 1, abort_flag, p.err)) {
                 ok = false;
@@ -332,6 +293,65 @@ __global__ void __launch_bounds__(kThreads, 1) k_contract(const __grid_constant_
                 __syncwarp();
             }
         }
+    } else if (MODE == CMODE_X) {
+        // ------------------------------------------------------------ gather warps
+        const int tt = threadIdx.x - 192;    // 0..127
+        uint32_t g = 0;
+        int pend_s = -1;                     // stage whose copies are not yet signalled
+        bool ok = true;
+        for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x) {
+            const int tile = item / p.splits, split = item % p.splits;
+            const int kc0 = split * p.kc_per_item;
+            const int kc1 = min(kc0 + p.kc_per_item, kc_total);
+            const int64_t r0 = tile_row0(tile, p.reorder, p.batches, p.seq_len);
+            const bool pe_tile = p.has_pe && !p.has_pos && (r0 % p.seq_len) + BM <= p.seq_len;
+            // element offsets of this thread's 8 rows in T_fixed and P (invalid
+            // ids / positions read row 0; the epilogue zeroes those rows)
+            int64_t trow[8], prow[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int64_t t = r0 + (tt >> 3) + 16 * u;
+                int64_t id = 0, ps = 0;
+                if (t < p.rows) {
+                    id = p.ids[t];
+                    if (id < 0 || id >= p.vocab)
+                        id = 0;
+                    if (p.has_pe) {
+                        ps = p.has_pos ? (int64_t)p.pos[t] : t % p.seq_len;
+                        if (ps < 0 || ps >= p.seq_len)
+                            ps = 0;
+                    }
+                }
+                trow[u] = id * p.d;
+                prow[u] = ps * p.d;
+            }
+            for (int kc = kc0; kc < kc1; ++kc, ++g) {
+                const int s = g % S;
+                const uint32_t n = g / S;
+                if (!warp_wait(empty_b + 8 * s, (n & 1) ^ 1, abort_flag, p.err)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t tb = base + s * pl.stage_bytes + pl.a_bytes + pl.u_bytes;
+                gather_tile_async(tb, p.tok, trow, (int64_t)kc * BK, p.d, tt);
+                if (p.has_pe && !pe_tile)
+                    gather_tile_async(tb + pl.raw_bytes, p.pe, prow, (int64_t)kc * BK, p.d, tt);
+                cp_async_commit();
+                if (pend_s >= 0) {   // the previous stage's copies have landed
+                    cp_async_wait1();
+                    fence_async_smem();
+                    __syncwarp();
+                    if (lane == 0)
+                        mbar_arrive(full_b + 8 * pend_s);
+                }
+                pend_s = s;
+            }
+        }
+        cp_async_wait0();
+        fence_async_smem();
+        __syncwarp();
+        if (pend_s >= 0 && lane == 0)
+            mbar_arrive(full_b + 8 * pend_s);
     }
 
     tc_fence_before();
@@ -347,22 +367,23 @@ __global__ void __launch_bounds__(kThreads, 1) k_contract(const __grid_constant_
 cudaError_t launch_contract(int mode, const ContractParams &p, int grid, cudaStream_t s)
 {
     const ContractPlan pl = contract_plan(mode, p.n_pad, p.k, p.has_pe, p.stages);
+    const int threads = contract_threads(mode);
     cudaError_t e;
     if (mode == CMODE_X) {
         e = cudaFuncSetAttribute(k_contract<CMODE_X>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  pl.total);
         if (e == cudaSuccess)
-            k_contract<CMODE_X><<<grid, kThreads, pl.total, s>>>(p);
+            k_contract<CMODE_X><<<grid, threads, pl.total, s>>>(p);
     } else if (mode == CMODE_G) {
         e = cudaFuncSetAttribute(k_contract<CMODE_G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  pl.total);
         if (e == cudaSuccess)
-            k_contract<CMODE_G><<<grid, kThreads, pl.total, s>>>(p);
+            k_contract<CMODE_G><<<grid, threads, pl.total, s>>>(p);
     } else {
         e = cudaFuncSetAttribute(k_contract<CMODE_W>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  pl.total);
         if (e == cudaSuccess)
-            k_contract<CMODE_W><<<grid, kThreads, pl.total, s>>>(p);
+            k_contract<CMODE_W><<<grid, threads, pl.total, s>>>(p);
     }
     if (e != cudaSuccess)
         return e;

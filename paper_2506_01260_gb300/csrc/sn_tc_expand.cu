@@ -6,10 +6,9 @@
 //
 // A work item is one 128-row tile and a run of 64-column output blocks.
 //   warp 0     TMA producer: per block, the 64 rows of the B operand (U, or
-//              A^T; 128-byte swizzled) and, for the reconstruction, the gathered
-//              T_fixed rows (tile::gather4, unswizzled) and the positional rows
-//              (one swizzled tile when the positions are contiguous, else
-//              gathered); per item, the A operand when it comes from a tensor map;
+//              A^T) and, for the reconstruction with contiguous positions, the
+//              positional tile; per item, the A operand when it comes from a
+//              tensor map (all 128-byte swizzled);
 //   warp 1     TMEM allocation and tcgen05.mma into a double-buffered fp32
 //              accumulator (M = 128, N = 64): C U^T over K = k padded to 16,
 //              then, for the reconstruction, + T_fixed rows . I + P rows . I
@@ -19,8 +18,9 @@
 //              operand (zero-padded); per block, drain the accumulator, round
 //              once to bf16 into a swizzled staging tile and TMA-store each
 //              warp's 32 rows (rows past the end are clipped by the map);
-//   warps 6-9  (reconstruction only) build the identity, then rewrite each
-//              block's gathered rows into the swizzled operand layout.
+//   warps 6-9  (reconstruction only) build the identity, then gather each
+//              block's T_fixed rows (and non-contiguous positional rows) with
+//              16-byte cp.async copies straight into their swizzled positions.
 // Every wait is bounded (SN_EBIT_TIMEOUT); an aborting CTA drains its copies
 // and MMAs and frees TMEM before it returns.
 #include "sn_tc.cuh"
@@ -45,7 +45,7 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
     const uint32_t a_s = base, id_s = base + pl.a_bytes;
     const uint32_t stage0 = base + pl.a_bytes + pl.id_bytes;
     const uint32_t bar = base + pl.bar_off;
-    const uint32_t full_b = bar, empty_b = bar + 8 * S, tready_b = bar + 16 * S;
+    const uint32_t full_b = bar, empty_b = bar + 8 * S;
     const uint32_t accf_b = bar + 24 * S, acce_b = accf_b + 16;
     const uint32_t afull_b = acce_b + 16, aempty_b = afull_b + 8, drain_b = aempty_b + 8;
     const uint32_t idready_b = drain_b + 8;
@@ -56,9 +56,8 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
-            mbar_init(full_b + 8 * s, 1);
+            mbar_init(full_b + 8 * s, GATHER ? 1 + 4 : 1);
             mbar_init(empty_b + 8 * s, 4);
-            mbar_init(tready_b + 8 * s, 4);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(accf_b + 8 * b, 1);
@@ -85,13 +84,8 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
             tma_prefetch(&p.mapB);
             if (AMODE == AMODE_TMA)
                 tma_prefetch(&p.mapA);
-            if (GATHER) {
-                tma_prefetch(&p.mapTok);
-                if (p.has_pe) {
-                    tma_prefetch(&p.mapPE);
-                    tma_prefetch(&p.mapPEg);
-                }
-            }
+            if (GATHER && p.has_pe)
+                tma_prefetch(&p.mapPE);
         }
         uint32_t g = 0, it = 0;
         bool ok = true;
@@ -111,28 +105,9 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                 }
                 __syncwarp();
             }
-            int rid[4] = {0, 0, 0, 0}, rps[4] = {0, 0, 0, 0};
-            bool pe_tile = false;
-            if (GATHER) {
-#pragma unroll
-                for (int r = 0; r < 4; ++r) {
-                    const int64_t t = r0 + 4 * lane + r;
-                    int id = 0, ps = 0;
-                    if (t < p.rows) {
-                        id = p.ids[t];
-                        if (id < 0 || id >= p.vocab)
-                            id = 0;                       // row zeroed by the epilogue
-                        if (p.has_pe) {
-                            ps = p.has_pos ? p.pos[t] : (int)(t % p.seq_len);
-                            if (ps < 0 || ps >= p.seq_len)
-                                ps = 0;
-                        }
-                    }
-                    rid[r] = id;
-                    rps[r] = ps;
-                }
-                pe_tile = p.has_pe && !p.has_pos && (r0 % p.seq_len) + BM <= p.seq_len;
-            }
+            const bool pe_tile =
+                GATHER && p.has_pe && !p.has_pos && (r0 % p.seq_len) + BM <= p.seq_len;
+            const uint32_t tx = pl.b_bytes + (pe_tile ? kTile : 0);
             for (int blk = blk0; blk < blk1; ++blk, ++g) {
                 const int s = g % S;
                 const uint32_t n = g / S;
@@ -142,23 +117,15 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                 }
                 const uint32_t st = stage0 + s * pl.stage_bytes;
                 const uint32_t fb = full_b + 8 * s;
-                if (lane == 0)
-                    mbar_arrive_tx(fb, pl.tx_bytes);
-                __syncwarp();
                 if (lane == 0) {
+                    mbar_arrive_tx(fb, tx);
                     for (int a = 0; a < p.katoms; ++a)
                         tma_load_2d(st + a * (BN * 128), &p.mapB, a * 64, blk * BN, fb);
-                    if (GATHER && pe_tile)
+                    if (pe_tile)
                         tma_load_2d(st + pl.b_bytes + kTile, &p.mapPE, blk * BN,
                                     (int)(r0 % p.seq_len), fb);
                 }
-                if (GATHER) {
-                    tma_gather4(st + pl.b_bytes + lane * 512, &p.mapTok, blk * BN, rid[0], rid[1],
-                                rid[2], rid[3], fb);
-                    if (p.has_pe && !pe_tile)
-                        tma_gather4(st + pl.b_bytes + kTile + lane * 512, &p.mapPEg, blk * BN,
-                                    rps[0], rps[1], rps[2], rps[3], fb);
-                }
+                __syncwarp();
             }
         }
         if (!ok && lane == 0) {
@@ -201,11 +168,6 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                                  sdesc_sw128(st + a * (BN * 128) + off), idesc, kk > 0 ? 1u : 0u);
                     }
                     if (GATHER) {   // + T_fixed rows . I + P rows . I
-                        if (!mbar_wait(tready_b + 8 * s, n & 1, abort_flag, p.err)) {
-                            ok = false;
-                            break;
-                        }
-                        tc_fence_after();
                         const uint32_t tb = st + pl.b_bytes;
 #pragma unroll
                         for (int kk = 0; kk < BN / 16; ++kk) {
@@ -370,29 +332,60 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
         if (lane == 0)
             mbar_arrive(idready_b);
         uint32_t g = 0;
+        int pend_s = -1;                     // stage whose copies are not yet signalled
         bool ok = true;
         for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x) {
             const int tile = item / p.chunks, ch = item % p.chunks;
             const int blk0 = ch * p.bpi, blk1 = min(blk0 + p.bpi, p.nblk);
             const int64_t r0 = tile_row0(tile, p.reorder, p.batches, p.seq_len);
-            const bool pe_contig = p.has_pe && !p.has_pos && (r0 % p.seq_len) + BM <= p.seq_len;
+            const bool pe_tile = p.has_pe && !p.has_pos && (r0 % p.seq_len) + BM <= p.seq_len;
+            // element offsets of this thread's 8 rows in T_fixed and P (invalid
+            // ids / positions read row 0; the epilogue zeroes those rows)
+            int64_t trow[8], prow[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int64_t t = r0 + (tt >> 3) + 16 * u;
+                int64_t id = 0, ps = 0;
+                if (t < p.rows) {
+                    id = p.ids[t];
+                    if (id < 0 || id >= p.vocab)
+                        id = 0;
+                    if (p.has_pe) {
+                        ps = p.has_pos ? (int64_t)p.pos[t] : t % p.seq_len;
+                        if (ps < 0 || ps >= p.seq_len)
+                            ps = 0;
+                    }
+                }
+                trow[u] = id * p.ncols;
+                prow[u] = ps * p.ncols;
+            }
             for (int blk = blk0; blk < blk1; ++blk, ++g) {
                 const int s = g % S;
                 const uint32_t n = g / S;
-                if (!warp_wait(full_b + 8 * s, n & 1, abort_flag, p.err)) {
+                if (!warp_wait(empty_b + 8 * s, (n & 1) ^ 1, abort_flag, p.err)) {
                     ok = false;
                     break;
                 }
                 const uint32_t tb = stage0 + s * pl.stage_bytes + pl.b_bytes;
-                swizzle_rows_in_place(tb, tt);
-                if (p.has_pe && !pe_contig)
-                    swizzle_rows_in_place(tb + kTile, tt);
-                fence_async_smem();
-                __syncwarp();
-                if (lane == 0)
-                    mbar_arrive(tready_b + 8 * s);
+                gather_tile_async(tb, p.tok, trow, (int64_t)blk * BN, p.ncols, tt);
+                if (p.has_pe && !pe_tile)
+                    gather_tile_async(tb + kTile, p.pe, prow, (int64_t)blk * BN, p.ncols, tt);
+                cp_async_commit();
+                if (pend_s >= 0) {   // the previous stage's copies have landed
+                    cp_async_wait1();
+                    fence_async_smem();
+                    __syncwarp();
+                    if (lane == 0)
+                        mbar_arrive(full_b + 8 * pend_s);
+                }
+                pend_s = s;
             }
         }
+        cp_async_wait0();
+        fence_async_smem();
+        __syncwarp();
+        if (pend_s >= 0 && lane == 0)
+            mbar_arrive(full_b + 8 * pend_s);
     }
 
     tc_fence_before();

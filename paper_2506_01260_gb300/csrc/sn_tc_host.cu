@@ -157,18 +157,15 @@ cudaError_t tc_compress(const sn_basis &b, const TcArgs &a, cudaStream_t s)
     const bool has_pe = a.gather && a.pe != nullptr;
     bool ok = map2d(&p.mapA, a.X, b.d, a.T, (uint64_t)b.d * 2, BK, BM, true) &&
               map2d(&p.mapU, b.ut16, b.d, b.n_pad, (uint64_t)b.d * 2, BK, b.n_pad, true);
-    if (ok && a.gather)
-        ok = map2d(&p.mapTok, a.tok, b.d, a.vocab, (uint64_t)b.d * 2, BK, 1, false);
-    else
-        p.mapTok = p.mapA;
     if (ok && has_pe)
-        ok = map2d(&p.mapPE, a.pe, b.d, a.seq_len, (uint64_t)b.d * 2, BK, BM, true) &&
-             map2d(&p.mapPEg, a.pe, b.d, a.seq_len, (uint64_t)b.d * 2, BK, 1, false);
+        ok = map2d(&p.mapPE, a.pe, b.d, a.seq_len, (uint64_t)b.d * 2, BK, BM, true);
     else
-        p.mapPE = p.mapPEg = p.mapA;
+        p.mapPE = p.mapA;
     if (!ok)
         return cudaErrorInvalidValue;
     const int mode = a.gather ? CMODE_X : CMODE_G;
+    p.tok = a.tok;
+    p.pe = has_pe ? a.pe : nullptr;
     p.ids = a.ids;
     p.pos = a.pos;
     p.C = a.C;
@@ -199,23 +196,18 @@ cudaError_t tc_decompress(const sn_basis &b, const TcArgs &a, __nv_bfloat16 *X_o
     ExpandParams p;
     std::memset(&p, 0, sizeof p);
     const bool has_pe = a.gather && a.pe != nullptr;
-    // gathered rows land unswizzled (every tile::gather4 destination is then
-    // 128-byte aligned) and are rewritten in shared memory; tiles are swizzled
     bool ok = map2d(&p.mapB, b.up16, b.k64, b.d, (uint64_t)b.k64 * 2, 64, BN, true) &&
               map2d(&p.mapOut, X_out, b.d / 8 * 8, a.T, (uint64_t)b.d * 2, 64, 32, true);
     p.mapA = p.mapB;
-    if (ok && a.gather)
-        ok = map2d(&p.mapTok, a.tok, b.d, a.vocab, (uint64_t)b.d * 2, 64, 1, false);
-    else
-        p.mapTok = p.mapB;
     if (ok && has_pe)
-        ok = map2d(&p.mapPE, a.pe, b.d, a.seq_len, (uint64_t)b.d * 2, 64, BM, true) &&
-             map2d(&p.mapPEg, a.pe, b.d, a.seq_len, (uint64_t)b.d * 2, 64, 1, false);
+        ok = map2d(&p.mapPE, a.pe, b.d, a.seq_len, (uint64_t)b.d * 2, 64, BM, true);
     else
-        p.mapPE = p.mapPEg = p.mapB;
+        p.mapPE = p.mapB;
     if (!ok)
         return cudaErrorInvalidValue;
     const int sms = sm_count(current_device());
+    p.tok = a.tok;
+    p.pe = has_pe ? a.pe : nullptr;
     p.C = a.C;
     p.ids = a.ids;
     p.pos = a.pos;
@@ -265,7 +257,7 @@ cudaError_t tc_project(const sn_basis &b, const __nv_bfloat16 *W, int64_t cols, 
     std::memset(&p, 0, sizeof p);
     bool ok = map2d(&p.mapA, W, cols, b.d, (uint64_t)ld * 2, BM, BK, false) &&
               map2d(&p.mapU, b.ut16, b.d, b.n_pad, (uint64_t)b.d * 2, BK, b.n_pad, true);
-    p.mapTok = p.mapPE = p.mapPEg = p.mapA;
+    p.mapPE = p.mapA;
     if (!ok)
         return cudaErrorInvalidValue;
     p.P = P;
@@ -297,7 +289,7 @@ cudaError_t tc_project(const sn_basis &b, const __nv_bfloat16 *W, int64_t cols, 
          map2d(&q.mapB, At, b.k64, cols, (uint64_t)b.k64 * 2, 64, BN, true) &&
          map2d(&q.mapOut, W_out, std::max<int64_t>(8, cols / 8 * 8), b.d, (uint64_t)ld * 2, 64,
                32, true);
-    q.mapTok = q.mapPE = q.mapPEg = q.mapB;
+    q.mapPE = q.mapB;
     if (!ok)
         return cudaErrorInvalidValue;
     q.err = b.err;

@@ -13,7 +13,6 @@ namespace tc {
 constexpr int BM = 128;          // rows (tokens / W columns / d rows) per tile = MMA M
 constexpr int BK = 64;           // contraction chunk: one 128-byte swizzle row of bf16
 constexpr int BN = 64;           // output columns per block of the expansion kernel
-constexpr int kThreads = 192;    // warp 0 TMA producer, warp 1 MMA, warps 2..5 compute
 constexpr uint32_t kSmemLimit = 232448;   // 227 KB per CTA
 constexpr uint32_t kTile = BM * 128;      // one [128 x 64] bf16 swizzled tile
 
@@ -23,9 +22,9 @@ enum { CMODE_G = 0, CMODE_X = 1, CMODE_W = 2 };
 struct ContractParams {
     CUtensorMap mapA;    // X or G [T, d] (SW128, box 64 x 128) | W [d, m] (plain, box 128 x 64)
     CUtensorMap mapU;    // U^T padded [n_pad, d] (SW128, box 64 x n_pad)
-    CUtensorMap mapTok;  // T_fixed [vocab, d] (plain, box 64 x 1, gather4)
-    CUtensorMap mapPE;   // P [seq_len, d] (SW128, box 64 x 128)
-    CUtensorMap mapPEg;  // P [seq_len, d] (plain, box 64 x 1, gather4)
+    CUtensorMap mapPE;   // P [seq_len, d] (SW128, box 64 x 128), contiguous positions
+    const __nv_bfloat16 *tok;   // T_fixed [vocab, d], rows gathered with cp.async
+    const __nv_bfloat16 *pe;    // P [seq_len, d], gathered when positions are not contiguous
     const int32_t *ids;
     const int32_t *pos;
     __nv_bfloat16 *C;    // [T, k] output (G, X modes)
@@ -42,6 +41,8 @@ struct ContractParams {
     int reorder, batches;
     int stages;
 };
+
+__host__ __device__ constexpr int contract_threads(int mode) { return mode == CMODE_X ? 320 : 192; }
 
 struct ContractPlan {
     uint32_t a_bytes, u_bytes, raw_bytes, pe_bytes, stage_bytes, cst_bytes, bar_off, total;
@@ -72,9 +73,9 @@ struct ExpandParams {
     CUtensorMap mapA;    // A by TMA: U padded [d, k64] (SW128, box 64 x 128)
     CUtensorMap mapB;    // B rows: U padded [d, k64] | A^T [m, k64] (SW128, box 64 x 64)
     CUtensorMap mapOut;  // output [rows, ncols] (SW128, box 64 x 32)
-    CUtensorMap mapTok;  // T_fixed (plain, box 64 x 1, gather4)
-    CUtensorMap mapPE;   // P (SW128, box 64 x 128)
-    CUtensorMap mapPEg;  // P (plain, box 64 x 1, gather4)
+    CUtensorMap mapPE;   // P (SW128, box 64 x 128), contiguous positions
+    const __nv_bfloat16 *tok;   // T_fixed [vocab, ncols], rows gathered with cp.async
+    const __nv_bfloat16 *pe;    // P [seq_len, ncols], gathered when positions are not contiguous
     const __nv_bfloat16 *C;   // A by repacking: [rows, k]
     __nv_bfloat16 *out;       // output base (ragged last columns are stored directly)
     int64_t out_ld;           // output leading dimension (elements)
