@@ -16,8 +16,10 @@
 //              added in fp32 inside the tensor core;
 //   warps 2-5  per item, repack the item's C rows into the swizzled K-major A
 //              operand (zero-padded); per block, drain the accumulator, round
-//              once to bf16 into a swizzled staging tile and TMA-store each
-//              warp's 32 rows (rows past the end are clipped by the map);
+//              once to bf16 into one of two swizzled staging tiles and
+//              TMA-store each warp's 32 rows (rows past the end are clipped by
+//              the map).  Stages are released by the MMA commit, so the stores
+//              never hold back the loads;
 //   warps 6-9  (reconstruction only) build the identity, then gather each
 //              block's T_fixed rows (and non-contiguous positional rows) with
 //              16-byte cp.async copies straight into their swizzled positions.
@@ -42,8 +44,8 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
 
     const int S = p.stages;
     const ExpandPlan pl = expand_plan(GATHER, p.katoms, p.has_pe, S);
-    const uint32_t a_s = base, id_s = base + pl.a_bytes;
-    const uint32_t stage0 = base + pl.a_bytes + pl.id_bytes;
+    const uint32_t a_s = base, id_s = base + pl.a_bytes, out_s = id_s + pl.id_bytes;
+    const uint32_t stage0 = out_s + pl.out_bytes;
     const uint32_t bar = base + pl.bar_off;
     const uint32_t full_b = bar, empty_b = bar + 8 * S;
     const uint32_t accf_b = bar + 24 * S, acce_b = accf_b + 16;
@@ -57,7 +59,7 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
             mbar_init(full_b + 8 * s, GATHER ? 1 + 4 : 1);
-            mbar_init(empty_b + 8 * s, 4);
+            mbar_init(empty_b + 8 * s, 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(accf_b + 8 * b, 1);
@@ -122,7 +124,7 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                     for (int a = 0; a < p.katoms; ++a)
                         tma_load_2d(st + a * (BN * 128), &p.mapB, a * 64, blk * BN, fb);
                     if (pe_tile)
-                        tma_load_2d(st + pl.b_bytes + kTile, &p.mapPE, blk * BN,
+                        tma_load_2d(st + pl.b_bytes + pl.t_bytes, &p.mapPE, blk * BN,
                                     (int)(r0 % p.seq_len), fb);
                 }
                 __syncwarp();
@@ -174,10 +176,11 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                             const uint64_t idd = sdesc_sw128(id_s + kk * 32);
                             mma_bf16(d_tmem, sdesc_sw128(tb + kk * 32), idd, idesc, 1u);
                             if (p.has_pe)
-                                mma_bf16(d_tmem, sdesc_sw128(tb + kTile + kk * 32), idd, idesc,
-                                         1u);
+                                mma_bf16(d_tmem, sdesc_sw128(tb + pl.t_bytes + kk * 32), idd,
+                                         idesc, 1u);
                         }
                     }
+                    mma_commit(empty_b + 8 * s);     // stage free once these MMAs finish
                     mma_commit(accf_b + 8 * b);
                 }
                 if (ok)
@@ -195,7 +198,6 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
         const int tt = threadIdx.x - 64;
         const int row = 32 * q + lane;
         uint32_t g = 0, it = 0;
-        int pend_s = -1;     // stage whose store may still be reading shared memory
         bool ok = true;
         for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++it) {
             const int tile = item / p.chunks, ch = item % p.chunks;
@@ -265,9 +267,13 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                 __syncwarp();
                 if (lane == 0)
                     mbar_arrive(acce_b + 8 * b);
-                // the output tile is staged over the block's T_fixed rows, which
-                // the MMA has finished reading
-                const uint32_t slot = stage0 + s * pl.stage_bytes + pl.b_bytes;
+                // output staging tile g & 1: the store issued from it two blocks
+                // ago must have finished reading it (one newer store may still be
+                // in flight)
+                const uint32_t slot = out_s + (g & 1) * kTile;
+                if (lane == 0)
+                    bulk_wait_read1();
+                __syncwarp();
 #pragma unroll
                 for (int c = 0; c < 8; ++c) {
                     uint4 o = make_uint4(pack_bf16(v[8 * c + 0], v[8 * c + 1]),
@@ -292,27 +298,15 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                 }
                 fence_async_smem();
                 __syncwarp();
-                if (lane == 0) {
-                    if (r0 + 32 * q < p.rows && c0 < p.ncols8) {
-                        tma_store_2d(&p.mapOut, slot + q * 4096, c0, (int)(r0 + 32 * q));
-                        bulk_commit();
-                    }
-                    // release the previous block's stage once its store has read
-                    // shared memory; this block's store stays in flight meanwhile
-                    bulk_wait_read1();
-                    if (pend_s >= 0)
-                        mbar_arrive(empty_b + 8 * pend_s);
+                if (lane == 0 && r0 + 32 * q < p.rows && c0 < p.ncols8) {
+                    tma_store_2d(&p.mapOut, slot + q * 4096, c0, (int)(r0 + 32 * q));
+                    bulk_commit();
                 }
-                pend_s = s;
                 __syncwarp();
             }
         }
-        if (lane == 0) {
-            bulk_wait_read0();
-            if (pend_s >= 0)
-                mbar_arrive(empty_b + 8 * pend_s);
+        if (lane == 0)
             bulk_wait_all0();
-        }
         __syncwarp();
     } else if (GATHER) {
         // ------------------------------------------------------------ row-layout warps
@@ -369,7 +363,7 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                 const uint32_t tb = stage0 + s * pl.stage_bytes + pl.b_bytes;
                 gather_tile_async(tb, p.tok, trow, (int64_t)blk * BN, p.ncols, tt);
                 if (p.has_pe && !pe_tile)
-                    gather_tile_async(tb + kTile, p.pe, prow, (int64_t)blk * BN, p.ncols, tt);
+                    gather_tile_async(tb + pl.t_bytes, p.pe, prow, (int64_t)blk * BN, p.ncols, tt);
                 cp_async_commit();
                 if (pend_s >= 0) {   // the previous stage's copies have landed
                     cp_async_wait1();

@@ -82,7 +82,7 @@ int contract_stages(int mode, int n_pad, int k, int has_pe)
 
 int expand_stages(bool gather, int katoms, int has_pe)
 {
-    int s = 6;
+    int s = 8;
     while (s > 2 && expand_plan(gather, katoms, has_pe, s).total > kSmemLimit)
         --s;
     return s;

@@ -93,25 +93,27 @@ struct ExpandParams {
 };
 
 struct ExpandPlan {
-    uint32_t a_bytes, id_bytes, b_bytes, out_bytes, pe_bytes, stage_bytes, bar_off, total,
-        tx_bytes;
+    uint32_t a_bytes, id_bytes, out_bytes, b_bytes, t_bytes, pe_bytes, stage_bytes, bar_off,
+        total;
 };
 
-// Shared memory of the expansion: A operand | identity (gather) | stages of
-// [B rows | T_fixed rows, later the output tile | positional rows] | barriers.
+// Shared memory of the expansion: A operand | identity (gather) | two output
+// staging tiles | stages of [B rows | T_fixed rows | positional rows] | barriers.
+// A stage is released by the MMA commit; outputs have their own ring, so the
+// stores never hold back the loads.
 __host__ __device__ inline ExpandPlan expand_plan(bool gather, int katoms, int has_pe,
                                                   int stages)
 {
     ExpandPlan p;
     p.a_bytes = (uint32_t)katoms * kTile;
     p.id_bytes = gather ? BN * 128 : 0;           // 64 x 64 bf16 identity, swizzled
+    p.out_bytes = 2 * kTile;
     p.b_bytes = (uint32_t)katoms * BN * 128;
-    p.out_bytes = kTile;
+    p.t_bytes = gather ? kTile : 0;
     p.pe_bytes = (gather && has_pe) ? kTile : 0;
-    p.stage_bytes = p.b_bytes + p.out_bytes + p.pe_bytes;
-    p.bar_off = p.a_bytes + p.id_bytes + (uint32_t)stages * p.stage_bytes;
+    p.stage_bytes = p.b_bytes + p.t_bytes + p.pe_bytes;
+    p.bar_off = p.a_bytes + p.id_bytes + p.out_bytes + (uint32_t)stages * p.stage_bytes;
     p.total = p.bar_off + 8 * (3 * stages + 8) + 16 + 1024;
-    p.tx_bytes = p.b_bytes + (gather ? p.out_bytes + p.pe_bytes : 0);
     return p;
 }
 
