@@ -9,18 +9,18 @@
 //              A^T) and, for the reconstruction with contiguous positions, the
 //              positional tile; per item, the A operand when it comes from a
 //              tensor map (all 128-byte swizzled);
-//   warp 1     TMEM allocation and tcgen05.mma into a double-buffered fp32
-//              accumulator (M = 128, N = 64): C U^T over K = k padded to 16,
+//   warp 1     TMEM allocation and tcgen05.mma into four fp32 accumulator
+//              buffers (M = 128, N = 64): C U^T over K = k padded to 16,
 //              then, for the reconstruction, + T_fixed rows . I + P rows . I
 //              with a resident 64 x 64 identity operand, so the embeddings are
 //              added in fp32 inside the tensor core;
-//   warps 2-5  per item, repack the item's C rows into the swizzled K-major A
-//              operand (zero-padded); per block, drain the accumulator, round
-//              once to bf16 into one of two swizzled staging tiles and
-//              TMA-store each warp's 32 rows (rows past the end are clipped by
-//              the map).  Stages are released by the MMA commit, so the stores
-//              never hold back the loads;
-//   warps 6-9  (reconstruction only) build the identity, then gather each
+//   warps 2-9  two epilogue groups taking alternate blocks: drain the
+//              accumulator, round once to bf16 into the group's swizzled
+//              staging tile and TMA-store each warp's 32 rows (rows past the end
+//              are clipped by the map); group 0 also repacks each item's C rows
+//              into the swizzled K-major A operand (zero-padded).  Stages are
+//              released by the MMA commit, so the stores never hold back loads;
+//   warps 10-13 (reconstruction only) build the identity, then gather each
 //              block's T_fixed rows (and non-contiguous positional rows) with
 //              16-byte cp.async copies straight into their swizzled positions.
 // Every wait is bounded (SN_EBIT_TIMEOUT); an aborting CTA drains its copies
@@ -48,20 +48,20 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
     const uint32_t stage0 = out_s + pl.out_bytes;
     const uint32_t bar = base + pl.bar_off;
     const uint32_t full_b = bar, empty_b = bar + 8 * S;
-    const uint32_t accf_b = bar + 24 * S, acce_b = accf_b + 16;
-    const uint32_t afull_b = acce_b + 16, aempty_b = afull_b + 8, drain_b = aempty_b + 8;
-    const uint32_t idready_b = drain_b + 8;
-    uint32_t *tmem_slot = (uint32_t *)(smem + pl.bar_off + 8 * (3 * S + 8));
+    const uint32_t accf_b = bar + 24 * S, acce_b = accf_b + 8 * kExpandAcc;
+    const uint32_t afull_b = acce_b + 8 * kExpandAcc, aempty_b = afull_b + 8;
+    const uint32_t drain_b = aempty_b + 8, idready_b = drain_b + 8;
+    uint32_t *tmem_slot = (uint32_t *)(smem + pl.bar_off + 8 * (3 * S + 12));
     volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    constexpr uint32_t kTmemCols = 2 * BN;
+    constexpr uint32_t kTmemCols = kExpandAcc * BN;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
             mbar_init(full_b + 8 * s, GATHER ? 1 + 4 : 1);
             mbar_init(empty_b + 8 * s, 1);
         }
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < kExpandAcc; ++b) {
             mbar_init(accf_b + 8 * b, 1);
             mbar_init(acce_b + 8 * b, 4);
         }
@@ -155,7 +155,7 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                 tc_fence_after();
                 for (int blk = blk0; blk < blk1; ++blk, ++g) {
                     const int s = g % S;
-                    const uint32_t n = g / S, b = g & 1, nb = g >> 1;
+                    const uint32_t n = g / S, b = g % kExpandAcc, nb = g / kExpandAcc;
                     if (!mbar_wait(full_b + 8 * s, n & 1, abort_flag, p.err) ||
                         !mbar_wait(acce_b + 8 * b, (nb & 1) ^ 1, abort_flag, p.err)) {
                         ok = false;
@@ -192,10 +192,11 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
             }
         }
         __syncwarp();
-    } else if (warp < 6) {
-        // ------------------------------------------------------------ epilogue warps
+    } else if (warp < 10) {
+        // ------------------------------------------------------------ epilogue groups
         const int q = warp & 3;
-        const int tt = threadIdx.x - 64;
+        const int grp = (warp - 2) >> 2;     // blocks g with g % 2 == grp
+        const int tt = threadIdx.x - 64;     // group 0 only: 0..127
         const int row = 32 * q + lane;
         uint32_t g = 0, it = 0;
         bool ok = true;
@@ -203,7 +204,7 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
             const int tile = item / p.chunks, ch = item % p.chunks;
             const int blk0 = ch * p.bpi, blk1 = min(blk0 + p.bpi, p.nblk);
             const int64_t r0 = tile_row0(tile, p.reorder, p.batches, p.seq_len);
-            if (AMODE == AMODE_REPACK) {
+            if (AMODE == AMODE_REPACK && grp == 0) {
                 // A operand: rows r0 .. r0+127 of C, zero-padded to katoms * 64 columns
                 if (!warp_wait(aempty_b, (it & 1) ^ 1, abort_flag, p.err)) {
                     ok = false;
@@ -250,8 +251,9 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                 }
             }
             for (int blk = blk0; blk < blk1; ++blk, ++g) {
-                const int s = g % S;
-                const uint32_t b = g & 1, nb = g >> 1;
+                if ((int)(g & 1) != grp)
+                    continue;
+                const uint32_t b = g % kExpandAcc, nb = g / kExpandAcc;
                 if (!warp_wait(accf_b + 8 * b, nb & 1, abort_flag, p.err)) {
                     ok = false;
                     break;
@@ -267,12 +269,11 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                 __syncwarp();
                 if (lane == 0)
                     mbar_arrive(acce_b + 8 * b);
-                // output staging tile g & 1: the store issued from it two blocks
-                // ago must have finished reading it (one newer store may still be
-                // in flight)
-                const uint32_t slot = out_s + (g & 1) * kTile;
+                // this group's staging tile: the warp's previous store from it
+                // must have finished reading it
+                const uint32_t slot = out_s + grp * kTile;
                 if (lane == 0)
-                    bulk_wait_read1();
+                    bulk_wait_read0();
                 __syncwarp();
 #pragma unroll
                 for (int c = 0; c < 8; ++c) {
@@ -309,8 +310,8 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
             bulk_wait_all0();
         __syncwarp();
     } else if (GATHER) {
-        // ------------------------------------------------------------ row-layout warps
-        const int tt = threadIdx.x - 192;    // 0..127
+        // ------------------------------------------------------------ gather warps
+        const int tt = threadIdx.x - 320;    // 0..127
         // identity B operand: 64 rows (N) x 64 columns (K), swizzled
 #pragma unroll
         for (int u = 0; u < 4; ++u) {

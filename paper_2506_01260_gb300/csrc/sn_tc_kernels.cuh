@@ -107,17 +107,20 @@ __host__ __device__ inline ExpandPlan expand_plan(bool gather, int katoms, int h
     ExpandPlan p;
     p.a_bytes = (uint32_t)katoms * kTile;
     p.id_bytes = gather ? BN * 128 : 0;           // 64 x 64 bf16 identity, swizzled
-    p.out_bytes = 2 * kTile;
+    p.out_bytes = 2 * kTile;                      // one staging tile per epilogue group
     p.b_bytes = (uint32_t)katoms * BN * 128;
     p.t_bytes = gather ? kTile : 0;
     p.pe_bytes = (gather && has_pe) ? kTile : 0;
     p.stage_bytes = p.b_bytes + p.t_bytes + p.pe_bytes;
     p.bar_off = p.a_bytes + p.id_bytes + p.out_bytes + (uint32_t)stages * p.stage_bytes;
-    p.total = p.bar_off + 8 * (3 * stages + 8) + 16 + 1024;
+    p.total = p.bar_off + 8 * (3 * stages + 12) + 16 + 1024;
     return p;
 }
 
-__host__ __device__ constexpr int expand_threads(bool gather) { return gather ? 320 : 192; }
+// warp 0 producer, warp 1 MMA, warps 2-5 and 6-9 two epilogue groups
+// (alternate blocks), warps 10-13 row gathers (reconstruction only)
+__host__ __device__ constexpr int expand_threads(bool gather) { return gather ? 448 : 320; }
+constexpr int kExpandAcc = 4;     // TMEM accumulator buffers of BN columns
 
 // Row tile -> first row.  With `reorder`, tiles run position-block-major so the
 // b sequences of a batch that share positional rows are processed together
