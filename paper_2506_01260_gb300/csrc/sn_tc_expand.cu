@@ -16,10 +16,10 @@
 //              added in fp32 inside the tensor core;
 //   warps 2-9  two epilogue groups taking alternate blocks: drain the
 //              accumulator, round once to bf16 into the group's swizzled
-//              staging tile and TMA-store each warp's 32 rows (rows past the end
-//              are clipped by the map); group 0 also repacks each item's C rows
-//              into the swizzled K-major A operand (zero-padded).  Stages are
-//              released by the MMA commit, so the stores never hold back loads;
+//              staging tile and write each warp's 32 rows with coalesced
+//              16-byte stores (the TMA unit is left to the loads); group 0 also
+//              repacks each item's C rows into the swizzled K-major A operand
+//              (zero-padded).  Stages are released by the MMA commit;
 //   warps 10-13 (reconstruction only) build the identity, then gather each
 //              block's T_fixed rows (and non-contiguous positional rows) with
 //              16-byte cp.async copies straight into their swizzled positions.
@@ -269,12 +269,10 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                 __syncwarp();
                 if (lane == 0)
                     mbar_arrive(acce_b + 8 * b);
-                // this group's staging tile: the warp's previous store from it
-                // must have finished reading it
+                // stage the rounded tile in this group's swizzled staging tile (the
+                // warp touches only its own 32 rows), then write it out with
+                // coalesced 16-byte stores: a quarter-warp per 128-byte row segment
                 const uint32_t slot = out_s + grp * kTile;
-                if (lane == 0)
-                    bulk_wait_read0();
-                __syncwarp();
 #pragma unroll
                 for (int c = 0; c < 8; ++c) {
                     uint4 o = make_uint4(pack_bf16(v[8 * c + 0], v[8 * c + 1]),
@@ -285,9 +283,8 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                         o = make_uint4(0, 0, 0, 0);
                     sts128(slot + sw128(row, c), o);
                 }
-                // Columns past the 8-aligned width of the output map (a TMA store
-                // clips the inner dimension only to 16 bytes) are written directly.
                 const int c0 = blk * BN;
+                // columns past the 8-aligned width are written element by element
                 if (!GATHER && c0 + BN > p.ncols8 && p.ncols > p.ncols8) {
                     const int64_t t = r0 + row;
                     if (t < p.rows) {
@@ -297,18 +294,21 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                                 p.out[t * p.out_ld + c0 + e] = __float2bfloat16_rn(v[e]);
                     }
                 }
-                fence_async_smem();
                 __syncwarp();
-                if (lane == 0 && r0 + 32 * q < p.rows && c0 < p.ncols8) {
-                    tma_store_2d(&p.mapOut, slot + q * 4096, c0, (int)(r0 + 32 * q));
-                    bulk_commit();
+                const int chunk = lane & 7;
+                const bool col_ok = c0 + 8 * chunk + 8 <= p.ncols8;
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const int rr = 32 * q + 4 * i + (lane >> 3);
+                    const int64_t t = r0 + rr;
+                    const uint4 o = lds128(slot + sw128(rr, chunk));
+                    if (col_ok && t < p.rows)
+                        *(uint4 *)(p.out + t * p.out_ld + c0 + 8 * chunk) = o;
                 }
                 __syncwarp();
             }
         }
-        if (lane == 0)
-            bulk_wait_all0();
-        __syncwarp();
+
     } else if (GATHER) {
         // ------------------------------------------------------------ gather warps
         const int tt = threadIdx.x - 320;    // 0..127
