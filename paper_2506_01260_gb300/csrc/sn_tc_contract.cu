@@ -20,6 +20,8 @@
 //   warps 6-9  CMODE_X: gather the T_fixed rows (and non-contiguous positional
 //              rows) with 16-byte cp.async copies straight into their swizzled
 //              positions, then fence toward the async proxy and arrive.
+// Each CTA walks an item's chunks starting at its own offset, so the CTAs' U^T
+// reads are spread over the L2 instead of converging on one slice.
 // Every wait is bounded; a wait that expires raises SN_EBIT_TIMEOUT and the
 // CTA drains its in-flight copies and MMAs, frees TMEM and returns.
 #include "sn_tc.cuh"
@@ -28,6 +30,13 @@
 namespace sn {
 namespace tc {
 namespace {
+
+// j-th chunk of an item: every CTA starts at a different chunk so that the
+// CTAs do not all read the same U^T chunk from one L2 slice at once.
+__device__ __forceinline__ int chunk_at(int kc0, int kc1, int j)
+{
+    return kc0 + (int)((j + blockIdx.x) % (kc1 - kc0));
+}
 
 template <int MODE>
 __global__ void __launch_bounds__(contract_threads(MODE), 1)
@@ -93,7 +102,8 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
                                  (r0 % p.seq_len) + BM <= p.seq_len;
             const uint32_t tx = MODE == CMODE_W ? pl.raw_bytes + pl.u_bytes
                                                 : pl.a_bytes + pl.u_bytes + (pe_tile ? kTile : 0);
-            for (int kc = kc0; kc < kc1; ++kc, ++g) {
+            for (int j = 0; j < kc1 - kc0; ++j, ++g) {
+                const int kc = chunk_at(kc0, kc1, j);
                 const int s = g % S;
                 const uint32_t n = g / S;
                 if (!warp_wait(empty_b + 8 * s, (n & 1) ^ 1, abort_flag, p.err)) {
@@ -139,7 +149,7 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
                 }
                 tc_fence_after();
                 const uint32_t d_tmem = tmem + b * p.acc_stride;
-                for (int kc = kc0; kc < kc1; ++kc, ++g) {
+                for (int j = 0; j < kc1 - kc0; ++j, ++g) {
                     const int s = g % S;
                     const uint32_t n = g / S;
                     const uint32_t wb = (MODE == CMODE_W ? rr_b : full_b) + 8 * s;
@@ -154,7 +164,7 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
                     for (int kk = 0; kk < BK / 16; ++kk) {
                         const uint64_t bd = sdesc_sw128(ub + kk * 32);
                         mma_bf16(d_tmem, sdesc_sw128(st + kk * 32), bd, idesc,
-                                 (kc > kc0 || kk > 0) ? 1u : 0u);
+                                 (j > 0 || kk > 0) ? 1u : 0u);
                         if (MODE == CMODE_X) {   // - T_fixed[ids] U - P[pos] U
                             const uint32_t tb = ub + pl.u_bytes;
                             mma_bf16(d_tmem, sdesc_sw128(tb + kk * 32), bd, idesc_neg, 1u);
@@ -188,7 +198,7 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
             const int64_t r0 = MODE == CMODE_W ? (int64_t)tile * BM
                                                : tile_row0(tile, p.reorder, p.batches, p.seq_len);
             if (MODE == CMODE_W) {
-                for (int kc = kc0; kc < kc1; ++kc, ++g) {
+                for (int j = 0; j < kc1 - kc0; ++j, ++g) {
                     const int s = g % S;
                     const uint32_t n = g / S;
                     if (!warp_wait(full_b + 8 * s, n & 1, abort_flag, p.err)) {
@@ -325,7 +335,8 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
                 trow[u] = id * p.d;
                 prow[u] = ps * p.d;
             }
-            for (int kc = kc0; kc < kc1; ++kc, ++g) {
+            for (int j = 0; j < kc1 - kc0; ++j, ++g) {
+                const int kc = chunk_at(kc0, kc1, j);
                 const int s = g % S;
                 const uint32_t n = g / S;
                 if (!warp_wait(empty_b + 8 * s, (n & 1) ^ 1, abort_flag, p.err)) {

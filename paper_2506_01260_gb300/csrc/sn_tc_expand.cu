@@ -17,9 +17,11 @@
 //   warps 2-9  two epilogue groups taking alternate blocks: drain the
 //              accumulator, round once to bf16 into the group's swizzled
 //              staging tile and write each warp's 32 rows with coalesced
-//              16-byte stores (the TMA unit is left to the loads); group 0 also
-//              repacks each item's C rows into the swizzled K-major A operand
-//              (zero-padded).  Stages are released by the MMA commit;
+//              16-byte stores (the TMA unit is left to the loads); together the
+//              groups repack each item's C rows into the swizzled K-major A
+//              operand (zero-padded).  Stages are released by the MMA commit.
+// Each CTA walks an item's blocks starting at its own offset, so the CTAs'
+// B-operand reads are spread over the L2 instead of converging on one slice;
 //   warps 10-13 (reconstruction only) build the identity, then gather each
 //              block's T_fixed rows (and non-contiguous positional rows) with
 //              16-byte cp.async copies straight into their swizzled positions.
@@ -31,6 +33,14 @@
 namespace sn {
 namespace tc {
 namespace {
+
+// j-th block of an item: every CTA starts at a different block so that the
+// CTAs do not all read the same rows of the B operand from one L2 slice at once.
+__device__ __forceinline__ int block_at(int blk0, int blk1, int j)
+{
+    const int nb = blk1 - blk0;
+    return blk0 + (int)((j + blockIdx.x) % nb);
+}
 
 template <int AMODE, bool GATHER>
 __global__ void __launch_bounds__(expand_threads(GATHER), 1)
@@ -65,7 +75,7 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
             mbar_init(accf_b + 8 * b, 1);
             mbar_init(acce_b + 8 * b, 4);
         }
-        mbar_init(afull_b, AMODE == AMODE_REPACK ? 4 : 1);
+        mbar_init(afull_b, AMODE == AMODE_REPACK ? 8 : 1);
         mbar_init(aempty_b, 1);
         mbar_init(drain_b, 1);
         mbar_init(idready_b, 4);
@@ -110,7 +120,8 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
             const bool pe_tile =
                 GATHER && p.has_pe && !p.has_pos && (r0 % p.seq_len) + BM <= p.seq_len;
             const uint32_t tx = pl.b_bytes + (pe_tile ? kTile : 0);
-            for (int blk = blk0; blk < blk1; ++blk, ++g) {
+            for (int j = 0; j < blk1 - blk0; ++j, ++g) {
+                const int blk = block_at(blk0, blk1, j);
                 const int s = g % S;
                 const uint32_t n = g / S;
                 if (!warp_wait(empty_b + 8 * s, (n & 1) ^ 1, abort_flag, p.err)) {
@@ -153,7 +164,7 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                     break;
                 }
                 tc_fence_after();
-                for (int blk = blk0; blk < blk1; ++blk, ++g) {
+                for (int j = 0; j < blk1 - blk0; ++j, ++g) {
                     const int s = g % S;
                     const uint32_t n = g / S, b = g % kExpandAcc, nb = g / kExpandAcc;
                     if (!mbar_wait(full_b + 8 * s, n & 1, abort_flag, p.err) ||
@@ -196,7 +207,7 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
         // ------------------------------------------------------------ epilogue groups
         const int q = warp & 3;
         const int grp = (warp - 2) >> 2;     // blocks g with g % 2 == grp
-        const int tt = threadIdx.x - 64;     // group 0 only: 0..127
+        const int tt = 32 * ((warp - 2) & 3) + lane;   // 0..127 within the group
         const int row = 32 * q + lane;
         uint32_t g = 0, it = 0;
         bool ok = true;
@@ -204,33 +215,38 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
             const int tile = item / p.chunks, ch = item % p.chunks;
             const int blk0 = ch * p.bpi, blk1 = min(blk0 + p.bpi, p.nblk);
             const int64_t r0 = tile_row0(tile, p.reorder, p.batches, p.seq_len);
-            if (AMODE == AMODE_REPACK && grp == 0) {
-                // A operand: rows r0 .. r0+127 of C, zero-padded to katoms * 64 columns
+            if (AMODE == AMODE_REPACK) {
+                // A operand: rows r0 .. r0+127 of C, zero-padded to katoms * 64
+                // columns.  Both groups share it: thread (r, half) covers atom
+                // `half` (two atoms) or chunks 4 half .. 4 half + 3 (one atom) of
+                // row r, issuing all of its loads before the first use.
                 if (!warp_wait(aempty_b, (it & 1) ^ 1, abort_flag, p.err)) {
                     ok = false;
                     break;
                 }
-                const int64_t t = r0 + tt;
+                const int r = tt, half = grp;
+                const int64_t t = r0 + r;
+                const int a = p.katoms == 2 ? half : 0;
+                const int cbeg = p.katoms == 2 ? 0 : 4 * half;
+                const int jbeg = a * 64 + cbeg * 8;
                 const unsigned short *crow = (const unsigned short *)p.C + t * p.k;
-                for (int a = 0; a < p.katoms; ++a) {
-#pragma unroll 2
-                    for (int c = 0; c < 8; ++c) {
-                        uint32_t w[4];
+                uint32_t h[32];
 #pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const int j = a * 64 + c * 8 + 2 * e;
-                            uint32_t lo = 0, hi = 0;
-                            if (t < p.rows) {
-                                if (j < p.k)
-                                    lo = __ldg(crow + j);
-                                if (j + 1 < p.k)
-                                    hi = __ldg(crow + j + 1);
-                            }
-                            w[e] = lo | (hi << 16);
-                        }
-                        sts128(a_s + a * kTile + sw128(tt, c), make_uint4(w[0], w[1], w[2], w[3]));
-                    }
+                for (int e = 0; e < 32; ++e) {
+                    const int j0 = jbeg + 2 * e;
+                    // one atom covers 64 columns: with two atoms each thread takes
+                    // 32 words, with one atom 16 words
+                    const bool want = (p.katoms == 2 || e < 16) && t < p.rows;
+                    const uint32_t lo = (want && j0 < p.k) ? __ldg(crow + j0) : 0u;
+                    const uint32_t hi = (want && j0 + 1 < p.k) ? __ldg(crow + j0 + 1) : 0u;
+                    h[e] = lo | (hi << 16);
                 }
+                const int nchunks = p.katoms == 2 ? 8 : 4;
+#pragma unroll
+                for (int c = 0; c < 8; ++c)
+                    if (c < nchunks)
+                        sts128(a_s + a * kTile + sw128(r, cbeg + c),
+                               make_uint4(h[4 * c], h[4 * c + 1], h[4 * c + 2], h[4 * c + 3]));
                 fence_async_smem();
                 __syncwarp();
                 if (lane == 0)
@@ -250,9 +266,10 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                         atomicOr(p.err, SN_EBIT_BAD_ID);
                 }
             }
-            for (int blk = blk0; blk < blk1; ++blk, ++g) {
+            for (int j = 0; j < blk1 - blk0; ++j, ++g) {
                 if ((int)(g & 1) != grp)
                     continue;
+                const int blk = block_at(blk0, blk1, j);
                 const uint32_t b = g % kExpandAcc, nb = g / kExpandAcc;
                 if (!warp_wait(accf_b + 8 * b, nb & 1, abort_flag, p.err)) {
                     ok = false;
@@ -354,7 +371,8 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                 trow[u] = id * p.ncols;
                 prow[u] = ps * p.ncols;
             }
-            for (int blk = blk0; blk < blk1; ++blk, ++g) {
+            for (int j = 0; j < blk1 - blk0; ++j, ++g) {
+                const int blk = block_at(blk0, blk1, j);
                 const int s = g % S;
                 const uint32_t n = g / S;
                 if (!warp_wait(empty_b + 8 * s, (n & 1) ^ 1, abort_flag, p.err)) {
