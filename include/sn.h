@@ -117,6 +117,26 @@ sn_status sn_project_weight(sn_basis_t basis, sn_dtype dtype, const void *W, int
                             int64_t cols, int64_t ld, void *W_out, void *workspace,
                             size_t workspace_bytes, sn_stream_t stream);
 
+/* sn_project_weight for callers that cannot allocate device memory: no
+ * workspace argument, no allocation.  The paper has no counterpart; this is a
+ * convenience of the library.  Some callers cannot call cudaMalloc or hand out
+ * scratch at the point where they project a weight (for example a training
+ * runtime whose caching allocator already owns the device memory, or code that
+ * must not enter the CUDA allocator between its own synchronisation points).
+ * The scratch lives in a fixed file-scope device array of 32 MiB (33554432
+ * bytes) that every GPU loading this library holds until the process exits.
+ * Arguments, layout and results are those of sn_project_weight; bf16 only.
+ * Returns SN_ERR_UNSUPPORTED for SN_F32 and when sn_project_weight_workspace
+ * for `cols` exceeds 32 MiB.  The first call on a device (with that device
+ * current) looks up the array's device address; make that first call before
+ * any stream capture.  All calls share the one array: calls whose executions
+ * overlap on the GPU (other streams, other host threads) race and corrupt each
+ * other's results, so order them on one stream.  Each call writes every
+ * scratch element it reads before reading it; nothing is kept between calls. */
+sn_status sn_project_weight_noalloc(sn_basis_t basis, sn_dtype dtype, const void *W,
+                                    int64_t rows, int64_t cols, int64_t ld, void *W_out,
+                                    sn_stream_t stream);
+
 /* Bytes on the wire for T tokens: T * k * element size (Sec. 4.3: k/d of X). */
 sn_status sn_wire_bytes(sn_basis_t basis, sn_dtype dtype, int64_t T, size_t *bytes);
 

@@ -45,6 +45,7 @@ _sig("sn_compress_bwd", [_P, _ST, _P, _I64, _P, _P])
 _sig("sn_decompress_bwd", [_P, _ST, _P, _I64, _P, _P])
 _sig("sn_project_weight_workspace", [_P, _ST, _I64, ctypes.POINTER(_SZ)])
 _sig("sn_project_weight", [_P, _ST, _P, _I64, _I64, _I64, _P, _P, _SZ, _P])
+_sig("sn_project_weight_noalloc", [_P, _ST, _P, _I64, _I64, _I64, _P, _P])
 _sig("sn_wire_bytes", [_P, _ST, _I64, ctypes.POINTER(_SZ)])
 _sig("sn_wire_send", [_P, _P, _SZ, _P])
 _sig("sn_wire_recv", [_P, _P, _SZ, _P])
@@ -55,7 +56,8 @@ _sig("sn_status_string", [_ST], ctypes.c_char_p)
 #: every function the C header declares (checked against include/sn.h by tests)
 EXPORTS = ["sn_basis_create", "sn_basis_destroy", "sn_basis_shape", "sn_compress_fwd",
            "sn_decompress_fwd", "sn_compress_bwd", "sn_decompress_bwd",
-           "sn_project_weight_workspace", "sn_project_weight", "sn_wire_bytes", "sn_wire_send",
+           "sn_project_weight_workspace", "sn_project_weight", "sn_project_weight_noalloc",
+           "sn_wire_bytes", "sn_wire_send",
            "sn_wire_recv", "sn_check_errors", "sn_launch_count", "sn_status_string"]
 
 
@@ -242,6 +244,23 @@ def sn_project_weight(basis, W, out=None, workspace=None, stream=None):
     _check(_lib.sn_project_weight(basis.handle, _dtype(W), _ptr(W), rows, cols, ld, _ptr(out),
                                   _ptr(workspace), workspace.numel() * workspace.element_size(),
                                   _stream(stream)), "sn_project_weight")
+    return out
+
+
+def sn_project_weight_noalloc(basis, W, out, stream=None):
+    """W' = U (U^T W) like sn_project_weight, for callers that cannot allocate
+    device memory: the library's fixed 32 MiB device scratch array is used
+    instead of a workspace, and the caller provides `out` (may be W).  bf16
+    only.  Calls that overlap on the GPU share the scratch and race."""
+    _need(W, "W", torch.bfloat16, contiguous=False)
+    if W.dim() != 2 or W.shape[0] != basis.d or W.stride(1) != 1:
+        raise ValueError("W must be [d, cols] with unit column stride")
+    if out.stride() != W.stride() or out.shape != W.shape or out.dtype != W.dtype:
+        raise ValueError("out must have W's shape, strides and dtype")
+    rows, cols = W.shape
+    _check(_lib.sn_project_weight_noalloc(basis.handle, SN_BF16, _ptr(W), rows, cols,
+                                          W.stride(0), _ptr(out), _stream(stream)),
+           "sn_project_weight_noalloc")
     return out
 
 
