@@ -78,6 +78,30 @@ def algorithmic_bytes(T, d, k, n, u, m_cols, s=2):
     }
 
 
+def kernel_sources_sha1():
+    import glob
+    import hashlib
+    h = hashlib.sha1()
+    for p in sorted(glob.glob(os.path.join(ROOT, "paper_2506_01260_gb300", "csrc", "*.cu*"))):
+        h.update(os.path.basename(p).encode())
+        with open(p, "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
+def measured_traffic(call):
+    """DRAM bytes per launch of `call` from the committed ncu capture, or None
+    when the kernel sources changed since the counters were taken."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        t = json.load(f)
+    if t.get("sources_sha1") != kernel_sources_sha1():
+        return None
+    return t.get("per_launch_bytes", {}).get(call)
+
+
 # ---- clocks ---------------------------------------------------------------------
 
 class ClockSampler:
@@ -363,11 +387,7 @@ def run_ours(args, world, rank, local, pg):
         kernels[name] = {"ms": seg[name], "algorithmic_bytes": ab[name], "gbs": gbs,
                          "frac": gbs / hbm}
     dom = max(names, key=lambda nm: seg[nm])
-    traffic = None
-    tpath = os.path.join(ROOT, "profiles", "traffic.json")
-    if os.path.exists(tpath):
-        with open(tpath) as f:
-            traffic = json.load(f).get(dom)
+    traffic = measured_traffic(dom) if args.workload == WORKLOAD else None
 
     # ---- end to end through the C ABI with host buffers ----
     e2e_line = None
