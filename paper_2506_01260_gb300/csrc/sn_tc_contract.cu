@@ -149,17 +149,14 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
                 }
                 tc_fence_after();
                 const uint32_t d_tmem = tmem + b * p.acc_stride;
-                // Software-pipelined: the next chunk's barrier is waited on before
-                // this chunk's commit is issued, because a wait issued after a
-                // commit does not return until the committed MMAs complete.
-                const int nk = kc1 - kc0;
-                const uint32_t wbase = MODE == CMODE_W ? rr_b : full_b;
-                if (!mbar_wait(wbase + 8 * (g % S), (g / S) & 1, abort_flag, p.err)) {
-                    ok = false;
-                    break;
-                }
-                for (int j = 0; j < nk; ++j, ++g) {
+                for (int j = 0; j < kc1 - kc0; ++j, ++g) {
                     const int s = g % S;
+                    const uint32_t n = g / S;
+                    const uint32_t wb = (MODE == CMODE_W ? rr_b : full_b) + 8 * s;
+                    if (!mbar_wait(wb, n & 1, abort_flag, p.err)) {
+                        ok = false;
+                        break;
+                    }
                     tc_fence_after();
                     const uint32_t st = base + s * pl.stage_bytes;
                     const uint32_t ub = st + pl.a_bytes;
@@ -176,20 +173,7 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
                                          idesc_neg, 1u);
                         }
                     }
-                    // (the gather warps signal a stage one stage late, so looking
-                    // ahead needs at least three stages)
-                    const bool ahead = j + 1 < nk && (MODE != CMODE_X || S >= 3);
-                    if (ahead &&
-                        !mbar_wait(wbase + 8 * ((g + 1) % S), ((g + 1) / S) & 1, abort_flag, p.err))
-                        ok = false;
                     mma_commit(empty_b + 8 * s);
-                    if (!ok)
-                        break;
-                    if (j + 1 < nk && !ahead &&
-                        !mbar_wait(wbase + 8 * ((g + 1) % S), ((g + 1) / S) & 1, abort_flag, p.err)) {
-                        ok = false;
-                        break;
-                    }
                 }
                 if (ok)
                     mma_commit(accf_b + 8 * b);

@@ -164,24 +164,14 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                     break;
                 }
                 tc_fence_after();
-                // Software-pipelined: the barriers of block j + 1 are waited on
-                // before block j's commits are issued, because a wait issued after
-                // a commit does not return until the committed MMAs complete.
-                const int nb_item = blk1 - blk0;
-                auto ready = [&](uint32_t gg) {
-                    const int ss = gg % S;
-                    const uint32_t bb = gg % kExpandAcc;
-                    return mbar_wait(full_b + 8 * ss, (gg / S) & 1, abort_flag, p.err) &&
-                           mbar_wait(acce_b + 8 * bb, ((gg / kExpandAcc) & 1) ^ 1, abort_flag,
-                                     p.err);
-                };
-                if (!ready(g)) {
-                    ok = false;
-                    break;
-                }
-                for (int j = 0; j < nb_item; ++j, ++g) {
+                for (int j = 0; j < blk1 - blk0; ++j, ++g) {
                     const int s = g % S;
-                    const uint32_t b = g % kExpandAcc;
+                    const uint32_t n = g / S, b = g % kExpandAcc, nb = g / kExpandAcc;
+                    if (!mbar_wait(full_b + 8 * s, n & 1, abort_flag, p.err) ||
+                        !mbar_wait(acce_b + 8 * b, (nb & 1) ^ 1, abort_flag, p.err)) {
+                        ok = false;
+                        break;
+                    }
                     tc_fence_after();
                     const uint32_t st = stage0 + s * pl.stage_bytes;
                     const uint32_t d_tmem = tmem + b * BN;
@@ -201,20 +191,8 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                                          idesc, 1u);
                         }
                     }
-                    // (the gather warps signal a stage one stage late, so looking
-                    // ahead needs at least three stages)
-                    const bool more = j + 1 < nb_item;
-                    const bool ahead = more && (!GATHER || S >= 3);
-                    if (ahead && !ready(g + 1))
-                        ok = false;
                     mma_commit(empty_b + 8 * s);     // stage free once these MMAs finish
                     mma_commit(accf_b + 8 * b);
-                    if (!ok)
-                        break;
-                    if (more && !ahead && !ready(g + 1)) {
-                        ok = false;
-                        break;
-                    }
                 }
                 if (ok)
                     mma_commit(aempty_b);
