@@ -9,14 +9,14 @@
 //   warp 0     TMA producer: the X/G tile (or raw W tile), the U^T chunk and,
 //              when a tile's positions are contiguous, the positional tile;
 //   warp 1     allocates TMEM and issues tcgen05.mma (M = 128, N = k padded
-//              to 16, K = 16) into a double-buffered fp32 accumulator;
-//   warps 2-5  CMODE_X: R = X - T_fixed rows - P rows in place (the three
-//              tiles share the swizzled layout, so this is elementwise; fp32
-//              arithmetic, one rounding of R to bf16), which keeps the tensor
-//              core at one MMA per K-step; CMODE_W: transpose the raw W tile
-//              into the K-major A operand; then drain the accumulator
-//              (tcgen05.ld), round once to bf16 and store each warp's 32 rows
-//              of C as one contiguous slab (CMODE_W: fp32 partial rows);
+//              to 16, K = 16) into a double-buffered fp32 accumulator.  CMODE_X
+//              accumulates X U - T_fixed[ids] U - P[pos] U: three MMAs per
+//              K-step, the embedding terms with the descriptor's negate-A bit,
+//              so the residual is never rounded;
+//   warps 2-5  CMODE_W: transpose the raw W tile into the K-major A operand;
+//              then drain the accumulator (tcgen05.ld), round once to bf16 and
+//              store each warp's 32 rows of C as one contiguous slab (CMODE_W:
+//              fp32 partial rows);
 //   warps 6-9  CMODE_X: gather the T_fixed rows (and non-contiguous positional
 //              rows) with 16-byte cp.async copies straight into their swizzled
 //              positions, then fence toward the async proxy and arrive.
@@ -36,11 +36,6 @@ namespace {
 __device__ __forceinline__ int chunk_at(int kc0, int kc1, int j)
 {
     return kc0 + (int)((j + blockIdx.x) % (kc1 - kc0));
-}
-
-__device__ __forceinline__ uint32_t sub3(uint32_t x, uint32_t t, uint32_t e)
-{
-    return pack_bf16(bf_lo(x) - bf_lo(t) - bf_lo(e), bf_hi(x) - bf_hi(t) - bf_hi(e));
 }
 
 template <int MODE>
@@ -140,6 +135,7 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
             const uint32_t idesc = idesc_bf16(BM, p.n_pad);
+            const uint32_t idesc_neg = idesc_bf16(BM, p.n_pad, true);
             uint32_t g = 0, it = 0;
             bool ok = true;
             for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++it) {
@@ -156,7 +152,7 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
                 for (int j = 0; j < kc1 - kc0; ++j, ++g) {
                     const int s = g % S;
                     const uint32_t n = g / S;
-                    const uint32_t wb = (MODE == CMODE_G ? full_b : rr_b) + 8 * s;
+                    const uint32_t wb = (MODE == CMODE_W ? rr_b : full_b) + 8 * s;
                     if (!mbar_wait(wb, n & 1, abort_flag, p.err)) {
                         ok = false;
                         break;
@@ -169,6 +165,13 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
                         const uint64_t bd = sdesc_sw128(ub + kk * 32);
                         mma_bf16(d_tmem, sdesc_sw128(st + kk * 32), bd, idesc,
                                  (j > 0 || kk > 0) ? 1u : 0u);
+                        if (MODE == CMODE_X) {   // - T_fixed[ids] U - P[pos] U
+                            const uint32_t tb = ub + pl.u_bytes;
+                            mma_bf16(d_tmem, sdesc_sw128(tb + kk * 32), bd, idesc_neg, 1u);
+                            if (p.has_pe)
+                                mma_bf16(d_tmem, sdesc_sw128(tb + pl.raw_bytes + kk * 32), bd,
+                                         idesc_neg, 1u);
+                        }
                     }
                     mma_commit(empty_b + 8 * s);
                 }
@@ -194,36 +197,6 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
             const int kc1 = min(kc0 + p.kc_per_item, kc_total);
             const int64_t r0 = MODE == CMODE_W ? (int64_t)tile * BM
                                                : tile_row0(tile, p.reorder, p.batches, p.seq_len);
-            if (MODE == CMODE_X) {
-                for (int j = 0; j < kc1 - kc0; ++j, ++g) {
-                    const int s = g % S;
-                    const uint32_t n = g / S;
-                    if (!warp_wait(full_b + 8 * s, n & 1, abort_flag, p.err)) {
-                        ok = false;
-                        break;
-                    }
-                    // R = X - T_fixed rows - P rows in place: all three tiles share
-                    // the swizzled layout, so the subtraction is elementwise; fp32
-                    // arithmetic, one rounding to the bf16 A operand
-                    const uint32_t st = base + s * pl.stage_bytes;
-                    const uint32_t tb = st + pl.a_bytes + pl.u_bytes, pb = tb + pl.raw_bytes;
-#pragma unroll 4
-                    for (int u = 0; u < 8; ++u) {
-                        const uint32_t off = (uint32_t)(tt + 128 * u) * 16;
-                        const uint4 x = lds128(st + off);
-                        const uint4 t = lds128(tb + off);
-                        const uint4 e = p.has_pe ? lds128(pb + off) : make_uint4(0, 0, 0, 0);
-                        sts128(st + off, make_uint4(sub3(x.x, t.x, e.x), sub3(x.y, t.y, e.y),
-                                                    sub3(x.z, t.z, e.z), sub3(x.w, t.w, e.w)));
-                    }
-                    fence_async_smem();
-                    __syncwarp();
-                    if (lane == 0)
-                        mbar_arrive(rr_b + 8 * s);
-                }
-                if (!ok)
-                    break;
-            }
             if (MODE == CMODE_W) {
                 for (int j = 0; j < kc1 - kc0; ++j, ++g) {
                     const int s = g % S;

@@ -10,19 +10,21 @@
 //              positional tile; per item, the A operand when it comes from a
 //              tensor map (all 128-byte swizzled);
 //   warp 1     TMEM allocation and tcgen05.mma into four fp32 accumulator
-//              buffers (M = 128, N = 64): C U^T over K = k padded to 16;
+//              buffers (M = 128, N = 64): C U^T over K = k padded to 16,
+//              then, for the reconstruction, + T_fixed rows . I + P rows . I
+//              with a resident 64 x 64 identity operand, so the embeddings are
+//              added in fp32 inside the tensor core;
 //   warps 2-9  two epilogue groups taking alternate blocks: drain the
-//              accumulator, add the block's positional and T_fixed rows in fp32
-//              (read from the swizzled stage, which the group then releases),
-//              round once to bf16 into the group's swizzled staging tile and write each warp's 32 rows with coalesced
+//              accumulator, round once to bf16 into the group's swizzled
+//              staging tile and write each warp's 32 rows with coalesced
 //              16-byte stores (the TMA unit is left to the loads); together the
 //              groups repack each item's C rows into the swizzled K-major A
 //              operand (zero-padded).  Stages are released by the MMA commit.
 // Each CTA walks an item's blocks starting at its own offset, so the CTAs'
 // B-operand reads are spread over the L2 instead of converging on one slice;
-//   warps 10-13 (reconstruction only) gather each block's T_fixed rows (and
-//              non-contiguous positional rows) with 16-byte cp.async copies
-//              straight into their swizzled positions.
+//   warps 10-13 (reconstruction only) build the identity, then gather each
+//              block's T_fixed rows (and non-contiguous positional rows) with
+//              16-byte cp.async copies straight into their swizzled positions.
 // Every wait is bounded (SN_EBIT_TIMEOUT); an aborting CTA drains its copies
 // and MMAs and frees TMEM before it returns.
 #include "sn_tc.cuh"
@@ -38,11 +40,6 @@ __device__ __forceinline__ int block_at(int blk0, int blk1, int j)
 {
     const int nb = blk1 - blk0;
     return blk0 + (int)((j + blockIdx.x) % nb);
-}
-
-__device__ __forceinline__ uint32_t add3(float a0, float a1, uint32_t pe, uint32_t te)
-{
-    return pack_bf16(a0 + bf_lo(pe) + bf_lo(te), a1 + bf_hi(pe) + bf_hi(te));
 }
 
 template <int AMODE, bool GATHER>
@@ -72,7 +69,7 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
             mbar_init(full_b + 8 * s, GATHER ? 1 + 4 : 1);
-            mbar_init(empty_b + 8 * s, GATHER ? 4 : 1);
+            mbar_init(empty_b + 8 * s, 1);
         }
         for (int b = 0; b < kExpandAcc; ++b) {
             mbar_init(accf_b + 8 * b, 1);
@@ -157,6 +154,8 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
             const uint32_t idesc = idesc_bf16(BM, BN);
             uint32_t g = 0, it = 0;
             bool ok = true;
+            if (GATHER && !mbar_wait(idready_b, 0, abort_flag, p.err))
+                ok = false;
             for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++it) {
                 const int ch = item % p.chunks;
                 const int blk0 = ch * p.bpi, blk1 = min(blk0 + p.bpi, p.nblk);
@@ -181,8 +180,18 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                         mma_bf16(d_tmem, sdesc_sw128(a_s + a * kTile + off),
                                  sdesc_sw128(st + a * (BN * 128) + off), idesc, kk > 0 ? 1u : 0u);
                     }
-                    if (!GATHER)   // stage free once these MMAs finish
-                        mma_commit(empty_b + 8 * s);
+                    if (GATHER) {   // + T_fixed rows . I + P rows . I
+                        const uint32_t tb = st + pl.b_bytes;
+#pragma unroll
+                        for (int kk = 0; kk < BN / 16; ++kk) {
+                            const uint64_t idd = sdesc_sw128(id_s + kk * 32);
+                            mma_bf16(d_tmem, sdesc_sw128(tb + kk * 32), idd, idesc, 1u);
+                            if (p.has_pe)
+                                mma_bf16(d_tmem, sdesc_sw128(tb + pl.t_bytes + kk * 32), idd,
+                                         idesc, 1u);
+                        }
+                    }
+                    mma_commit(empty_b + 8 * s);     // stage free once these MMAs finish
                     mma_commit(accf_b + 8 * b);
                 }
                 if (ok)
@@ -281,42 +290,15 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                 // warp touches only its own 32 rows), then write it out with
                 // coalesced 16-byte stores: a quarter-warp per 128-byte row segment
                 const uint32_t slot = out_s + grp * kTile;
-                if (GATHER) {
-                    // + P rows + T_fixed rows in fp32 (swizzled tiles: a thread reads
-                    // its own row, the quarter-warp's 8 rows hit 8 different banks),
-                    // then release the stage
-                    const int s = g % S;
-                    if (!warp_wait(full_b + 8 * s, (g / S) & 1, abort_flag, p.err)) {
-                        ok = false;
-                        break;
-                    }
-                    const uint32_t tb = stage0 + s * pl.stage_bytes + pl.b_bytes;
-                    uint4 o[8];
 #pragma unroll
-                    for (int c = 0; c < 8; ++c) {
-                        const uint32_t off = sw128(row, c);
-                        const uint4 tv = lds128(tb + off);
-                        const uint4 pv = p.has_pe ? lds128(tb + pl.t_bytes + off)
-                                                  : make_uint4(0, 0, 0, 0);
-                        o[c] = make_uint4(add3(v[8 * c + 0], v[8 * c + 1], pv.x, tv.x),
-                                          add3(v[8 * c + 2], v[8 * c + 3], pv.y, tv.y),
-                                          add3(v[8 * c + 4], v[8 * c + 5], pv.z, tv.z),
-                                          add3(v[8 * c + 6], v[8 * c + 7], pv.w, tv.w));
-                    }
-                    __syncwarp();
-                    if (lane == 0)
-                        mbar_arrive(empty_b + 8 * s);
-#pragma unroll
-                    for (int c = 0; c < 8; ++c)
-                        sts128(slot + sw128(row, c), bad ? make_uint4(0, 0, 0, 0) : o[c]);
-                } else {
-#pragma unroll
-                    for (int c = 0; c < 8; ++c)
-                        sts128(slot + sw128(row, c),
-                               make_uint4(pack_bf16(v[8 * c + 0], v[8 * c + 1]),
-                                          pack_bf16(v[8 * c + 2], v[8 * c + 3]),
-                                          pack_bf16(v[8 * c + 4], v[8 * c + 5]),
-                                          pack_bf16(v[8 * c + 6], v[8 * c + 7])));
+                for (int c = 0; c < 8; ++c) {
+                    uint4 o = make_uint4(pack_bf16(v[8 * c + 0], v[8 * c + 1]),
+                                         pack_bf16(v[8 * c + 2], v[8 * c + 3]),
+                                         pack_bf16(v[8 * c + 4], v[8 * c + 5]),
+                                         pack_bf16(v[8 * c + 6], v[8 * c + 7]));
+                    if (bad)
+                        o = make_uint4(0, 0, 0, 0);
+                    sts128(slot + sw128(row, c), o);
                 }
                 const int c0 = blk * BN;
                 // columns past the 8-aligned width are written element by element
@@ -347,6 +329,20 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
     } else if (GATHER) {
         // ------------------------------------------------------------ gather warps
         const int tt = threadIdx.x - 320;    // 0..127
+        // identity B operand: 64 rows (N) x 64 columns (K), swizzled
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int unit = tt + 128 * u, n = unit >> 3, c = unit & 7;
+            // row n holds bf16 1.0 at column n: chunk n / 8, element n % 8
+            const uint32_t one = (n & 1) ? 0x3F800000u : 0x00003F80u;
+            const int word = ((n >> 3) == c) ? ((n & 7) >> 1) : -1;
+            sts128(id_s + sw128(n, c), make_uint4(word == 0 ? one : 0u, word == 1 ? one : 0u,
+                                                  word == 2 ? one : 0u, word == 3 ? one : 0u));
+        }
+        fence_async_smem();
+        __syncwarp();
+        if (lane == 0)
+            mbar_arrive(idready_b);
         uint32_t g = 0;
         int pend_s = -1;                     // stage whose copies are not yet signalled
         bool ok = true;

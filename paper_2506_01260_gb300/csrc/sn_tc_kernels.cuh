@@ -97,17 +97,16 @@ struct ExpandPlan {
         total;
 };
 
-// Shared memory of the expansion: A operand | two output staging tiles |
-// stages of [B rows | T_fixed rows | positional rows] | barriers.  A stage is
-// released by the MMA commit (or, when the epilogue reads its gathered rows,
-// by the epilogue); outputs have their own staging, so stores never hold back
-// the loads.
+// Shared memory of the expansion: A operand | identity (gather) | two output
+// staging tiles | stages of [B rows | T_fixed rows | positional rows] | barriers.
+// A stage is released by the MMA commit; outputs have their own ring, so the
+// stores never hold back the loads.
 __host__ __device__ inline ExpandPlan expand_plan(bool gather, int katoms, int has_pe,
                                                   int stages)
 {
     ExpandPlan p;
     p.a_bytes = (uint32_t)katoms * kTile;
-    p.id_bytes = 0;
+    p.id_bytes = gather ? BN * 128 : 0;           // 64 x 64 bf16 identity, swizzled
     p.out_bytes = 2 * kTile;                      // one staging tile per epilogue group
     p.b_bytes = (uint32_t)katoms * BN * 128;
     p.t_bytes = gather ? kTile : 0;
