@@ -4,13 +4,14 @@
 //   decompress_bwd  G[t, :] = C[t, :] U^T                                 Sec. 4.4
 //   project (b)     W'[i, :] = U[i, :] A   with A = U^T W from the first pass
 //
-// A work item is one 128-row tile and a run of 64-column output blocks.
-//   warp 0     TMA producer: per block, the 64 rows of the B operand (U, or
+// A work item is one 128-row tile and a run of NB-column output blocks (NB = 64
+// for the reconstruction, 128 otherwise).
+//   warp 0     TMA producer: per block, the NB rows of the B operand (U, or
 //              A^T) and, for the reconstruction with contiguous positions, the
 //              positional tile; per item, the A operand when it comes from a
 //              tensor map (all 128-byte swizzled);
 //   warp 1     TMEM allocation and tcgen05.mma into four fp32 accumulator
-//              buffers (M = 128, N = 64): C U^T over K = k padded to 16,
+//              buffers (M = 128, N = NB): C U^T over K = k padded to 16,
 //              then, for the reconstruction, + T_fixed rows . I + P rows . I
 //              with a resident 64 x 64 identity operand, so the embeddings are
 //              added in fp32 inside the tensor core;
@@ -64,7 +65,9 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
     uint32_t *tmem_slot = (uint32_t *)(smem + pl.bar_off + 8 * (3 * S + 12));
     volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    constexpr uint32_t kTmemCols = kExpandAcc * BN;
+    constexpr int NB = expand_bn(GATHER);
+    static_assert(!GATHER || NB == BN, "the gathered rows and the identity are 64 wide");
+    constexpr uint32_t kTmemCols = kExpandAcc * NB;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
@@ -133,7 +136,7 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                 if (lane == 0) {
                     mbar_arrive_tx(fb, tx);
                     for (int a = 0; a < p.katoms; ++a)
-                        tma_load_2d(st + a * (BN * 128), &p.mapB, a * 64, blk * BN, fb);
+                        tma_load_2d(st + a * (NB * 128), &p.mapB, a * 64, blk * NB, fb);
                     if (pe_tile)
                         tma_load_2d(st + pl.b_bytes + pl.t_bytes, &p.mapPE, blk * BN,
                                     (int)(r0 % p.seq_len), fb);
@@ -151,7 +154,7 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
-            const uint32_t idesc = idesc_bf16(BM, BN);
+            const uint32_t idesc = idesc_bf16(BM, NB);
             uint32_t g = 0, it = 0;
             bool ok = true;
             if (GATHER && !mbar_wait(idready_b, 0, abort_flag, p.err))
@@ -174,11 +177,11 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                     }
                     tc_fence_after();
                     const uint32_t st = stage0 + s * pl.stage_bytes;
-                    const uint32_t d_tmem = tmem + b * BN;
+                    const uint32_t d_tmem = tmem + b * NB;
                     for (int kk = 0; kk < p.kmma; ++kk) {
                         const uint32_t a = kk >> 2, off = (kk & 3) * 32;
                         mma_bf16(d_tmem, sdesc_sw128(a_s + a * kTile + off),
-                                 sdesc_sw128(st + a * (BN * 128) + off), idesc, kk > 0 ? 1u : 0u);
+                                 sdesc_sw128(st + a * (NB * 128) + off), idesc, kk > 0 ? 1u : 0u);
                     }
                     if (GATHER) {   // + T_fixed rows . I + P rows . I
                         const uint32_t tb = st + pl.b_bytes;
@@ -276,49 +279,58 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                     break;
                 }
                 tc_fence_after();
-                float v[BN];
-                const uint32_t taddr = tmem + b * BN + ((uint32_t)(32 * q) << 16);
+                // drain the accumulator 64 columns at a time and stage the rounded
+                // values in this group's swizzled staging tile (one [128 x 64]
+                // atom per 64 columns; the warp touches only its own 32 rows)
+                const uint32_t slot = out_s + grp * (NB / 64) * kTile;
+                const int c0 = blk * NB;
 #pragma unroll
-                for (int i = 0; i < BN / 16; ++i)
-                    tmem_ld16(taddr + 16 * i, *(float(*)[16])(v + 16 * i));
-                tmem_ld_wait();
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0)
-                    mbar_arrive(acce_b + 8 * b);
-                // stage the rounded tile in this group's swizzled staging tile (the
-                // warp touches only its own 32 rows), then write it out with
-                // coalesced 16-byte stores: a quarter-warp per 128-byte row segment
-                const uint32_t slot = out_s + grp * kTile;
+                for (int h = 0; h < NB / 64; ++h) {
+                    float v[64];
+                    const uint32_t taddr = tmem + b * NB + 64 * h + ((uint32_t)(32 * q) << 16);
 #pragma unroll
-                for (int c = 0; c < 8; ++c) {
-                    uint4 o = make_uint4(pack_bf16(v[8 * c + 0], v[8 * c + 1]),
-                                         pack_bf16(v[8 * c + 2], v[8 * c + 3]),
-                                         pack_bf16(v[8 * c + 4], v[8 * c + 5]),
-                                         pack_bf16(v[8 * c + 6], v[8 * c + 7]));
-                    if (bad)
-                        o = make_uint4(0, 0, 0, 0);
-                    sts128(slot + sw128(row, c), o);
-                }
-                const int c0 = blk * BN;
-                // columns past the 8-aligned width are written element by element
-                if (!GATHER && c0 + BN > p.ncols8 && p.ncols > p.ncols8) {
-                    const int64_t t = r0 + row;
-                    if (t < p.rows) {
+                    for (int i = 0; i < 4; ++i)
+                        tmem_ld16(taddr + 16 * i, *(float(*)[16])(v + 16 * i));
+                    tmem_ld_wait();
+                    if (h == NB / 64 - 1) {
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0)
+                            mbar_arrive(acce_b + 8 * b);
+                    }
 #pragma unroll
-                        for (int e = 0; e < BN; ++e)
-                            if (c0 + e >= p.ncols8 && c0 + e < p.ncols)
-                                p.out[t * p.out_ld + c0 + e] = __float2bfloat16_rn(v[e]);
+                    for (int c = 0; c < 8; ++c) {
+                        uint4 o = make_uint4(pack_bf16(v[8 * c + 0], v[8 * c + 1]),
+                                             pack_bf16(v[8 * c + 2], v[8 * c + 3]),
+                                             pack_bf16(v[8 * c + 4], v[8 * c + 5]),
+                                             pack_bf16(v[8 * c + 6], v[8 * c + 7]));
+                        if (bad)
+                            o = make_uint4(0, 0, 0, 0);
+                        sts128(slot + h * kTile + sw128(row, c), o);
+                    }
+                    // columns past the 8-aligned width are written element by element
+                    const int ch0 = c0 + 64 * h;
+                    if (!GATHER && ch0 + 64 > p.ncols8 && p.ncols > p.ncols8) {
+                        const int64_t t = r0 + row;
+                        if (t < p.rows) {
+#pragma unroll
+                            for (int e = 0; e < 64; ++e)
+                                if (ch0 + e >= p.ncols8 && ch0 + e < p.ncols)
+                                    p.out[t * p.out_ld + ch0 + e] = __float2bfloat16_rn(v[e]);
+                        }
                     }
                 }
                 __syncwarp();
-                const int chunk = lane & 7;
+                // coalesced 16-byte stores: NB / 8 lanes per output row segment
+                constexpr int kCpr = NB / 8, kRpi = 32 / kCpr;
+                const int chunk = lane % kCpr;
                 const bool col_ok = c0 + 8 * chunk + 8 <= p.ncols8;
+                const uint32_t src = slot + (chunk >> 3) * kTile;
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const int rr = 32 * q + 4 * i + (lane >> 3);
+                for (int i = 0; i < 32 / kRpi; ++i) {
+                    const int rr = 32 * q + kRpi * i + lane / kCpr;
                     const int64_t t = r0 + rr;
-                    const uint4 o = lds128(slot + sw128(rr, chunk));
+                    const uint4 o = lds128(src + sw128(rr, chunk & 7));
                     if (col_ok && t < p.rows)
                         *(uint4 *)(p.out + t * p.out_ld + c0 + 8 * chunk) = o;
                 }

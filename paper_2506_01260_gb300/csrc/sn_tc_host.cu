@@ -196,7 +196,8 @@ cudaError_t tc_decompress(const sn_basis &b, const TcArgs &a, __nv_bfloat16 *X_o
     ExpandParams p;
     std::memset(&p, 0, sizeof p);
     const bool has_pe = a.gather && a.pe != nullptr;
-    bool ok = map2d(&p.mapB, b.up16, b.k64, b.d, (uint64_t)b.k64 * 2, 64, BN, true) &&
+    const int nb = expand_bn(a.gather);
+    bool ok = map2d(&p.mapB, b.up16, b.k64, b.d, (uint64_t)b.k64 * 2, 64, nb, true) &&
               map2d(&p.mapOut, X_out, b.d / 8 * 8, a.T, (uint64_t)b.d * 2, 64, 32, true);
     p.mapA = p.mapB;
     if (ok && has_pe)
@@ -224,7 +225,7 @@ cudaError_t tc_decompress(const sn_basis &b, const TcArgs &a, __nv_bfloat16 *X_o
     p.out_ld = b.d;
     p.ncols = b.d;
     p.ncols8 = b.d / 8 * 8;
-    p.nblk = (b.d + BN - 1) / BN;
+    p.nblk = (b.d + nb - 1) / nb;
     p.ntiles = (int)((a.T + BM - 1) / BM);
     split_blocks(p.ntiles, p.nblk, sms, &p.bpi, &p.chunks);
     tile_order(a.T, a.seq_len, has_pe, p.has_pos, &p.reorder, &p.batches);
@@ -286,7 +287,7 @@ cudaError_t tc_project(const sn_basis &b, const __nv_bfloat16 *W, int64_t cols, 
     ExpandParams q;
     std::memset(&q, 0, sizeof q);
     ok = map2d(&q.mapA, b.up16, b.k64, b.d, (uint64_t)b.k64 * 2, 64, BM, true) &&
-         map2d(&q.mapB, At, b.k64, cols, (uint64_t)b.k64 * 2, 64, BN, true) &&
+         map2d(&q.mapB, At, b.k64, cols, (uint64_t)b.k64 * 2, 64, BN_WIDE, true) &&
          map2d(&q.mapOut, W_out, std::max<int64_t>(8, cols / 8 * 8), b.d, (uint64_t)ld * 2, 64,
                32, true);
     q.mapPE = q.mapB;
@@ -303,7 +304,7 @@ cudaError_t tc_project(const sn_basis &b, const __nv_bfloat16 *W, int64_t cols, 
     q.out_ld = ld;
     q.ncols = (int)cols;
     q.ncols8 = (int)(cols / 8 * 8);
-    q.nblk = (int)((cols + BN - 1) / BN);
+    q.nblk = (int)((cols + BN_WIDE - 1) / BN_WIDE);
     q.ntiles = (b.d + BM - 1) / BM;
     split_blocks(q.ntiles, q.nblk, sms, &q.bpi, &q.chunks);
     q.stages = expand_stages(false, q.katoms, 0);

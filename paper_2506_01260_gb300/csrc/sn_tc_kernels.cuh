@@ -12,7 +12,8 @@ namespace tc {
 
 constexpr int BM = 128;          // rows (tokens / W columns / d rows) per tile = MMA M
 constexpr int BK = 64;           // contraction chunk: one 128-byte swizzle row of bf16
-constexpr int BN = 64;           // output columns per block of the expansion kernel
+constexpr int BN = 64;           // output columns per block of the reconstruction
+constexpr int BN_WIDE = 128;     // output columns per block of the plain expansion
 constexpr uint32_t kSmemLimit = 232448;   // 227 KB per CTA
 constexpr uint32_t kTile = BM * 128;      // one [128 x 64] bf16 swizzled tile
 
@@ -71,7 +72,7 @@ enum { AMODE_REPACK = 0, AMODE_TMA = 1 };
 
 struct ExpandParams {
     CUtensorMap mapA;    // A by TMA: U padded [d, k64] (SW128, box 64 x 128)
-    CUtensorMap mapB;    // B rows: U padded [d, k64] | A^T [m, k64] (SW128, box 64 x 64)
+    CUtensorMap mapB;    // B rows: U padded [d, k64] | A^T [m, k64] (SW128, box 64 x NB)
     CUtensorMap mapOut;  // output [rows, ncols] (SW128, box 64 x 32)
     CUtensorMap mapPE;   // P (SW128, box 64 x 128), contiguous positions
     const __nv_bfloat16 *tok;   // T_fixed [vocab, ncols], rows gathered with cp.async
@@ -97,6 +98,12 @@ struct ExpandPlan {
         total;
 };
 
+// Output columns per block (the MMA's N): the reconstruction keeps 64 so that a
+// stage still holds the gathered T_fixed and positional rows; the plain
+// expansion takes 128, which halves the MMA instructions and per-block
+// hand-offs and reads each A slice from shared memory once per 128 columns.
+__host__ __device__ constexpr int expand_bn(bool gather) { return gather ? BN : BN_WIDE; }
+
 // Shared memory of the expansion: A operand | identity (gather) | two output
 // staging tiles | stages of [B rows | T_fixed rows | positional rows] | barriers.
 // A stage is released by the MMA commit; outputs have their own ring, so the
@@ -105,10 +112,11 @@ __host__ __device__ inline ExpandPlan expand_plan(bool gather, int katoms, int h
                                                   int stages)
 {
     ExpandPlan p;
+    const uint32_t nb = (uint32_t)expand_bn(gather);
     p.a_bytes = (uint32_t)katoms * kTile;
     p.id_bytes = gather ? BN * 128 : 0;           // 64 x 64 bf16 identity, swizzled
-    p.out_bytes = 2 * kTile;                      // one staging tile per epilogue group
-    p.b_bytes = (uint32_t)katoms * BN * 128;
+    p.out_bytes = 2 * BM * nb * 2;                // one staging tile per epilogue group
+    p.b_bytes = (uint32_t)katoms * nb * 128;
     p.t_bytes = gather ? kTile : 0;
     p.pe_bytes = (gather && has_pe) ? kTile : 0;
     p.stage_bytes = p.b_bytes + p.t_bytes + p.pe_bytes;
@@ -120,7 +128,7 @@ __host__ __device__ inline ExpandPlan expand_plan(bool gather, int katoms, int h
 // warp 0 producer, warp 1 MMA, warps 2-5 and 6-9 two epilogue groups
 // (alternate blocks), warps 10-13 row gathers (reconstruction only)
 __host__ __device__ constexpr int expand_threads(bool gather) { return gather ? 448 : 320; }
-constexpr int kExpandAcc = 4;     // TMEM accumulator buffers of BN columns
+constexpr int kExpandAcc = 4;     // TMEM accumulator buffers of expand_bn() columns
 
 // Row tile -> first row.  With `reorder`, tiles run position-block-major so the
 // b sequences of a batch that share positional rows are processed together
