@@ -88,6 +88,16 @@ int expand_stages(bool gather, int katoms, int has_pe)
     return s;
 }
 
+// Two B stages; as many embedding stages as fit (at most 12).
+void recon_stages(int katoms, int has_pe, int *sb, int *se)
+{
+    *sb = 2;
+    int s = 12;
+    while (s > 2 && recon_plan(katoms, has_pe, *sb, s).total > kSmemLimit)
+        --s;
+    *se = s;
+}
+
 // Tiles ordered position-block-major when every sequence of the batch shares
 // the same positional rows in whole 128-row blocks.
 void tile_order(int64_t T, int seq_len, bool has_pe, bool has_pos, int *reorder, int *batches)
@@ -196,7 +206,7 @@ cudaError_t tc_decompress(const sn_basis &b, const TcArgs &a, __nv_bfloat16 *X_o
     ExpandParams p;
     std::memset(&p, 0, sizeof p);
     const bool has_pe = a.gather && a.pe != nullptr;
-    const int nb = expand_bn(a.gather);
+    const int nb = BN_WIDE;
     bool ok = map2d(&p.mapB, b.up16, b.k64, b.d, (uint64_t)b.k64 * 2, 64, nb, true) &&
               map2d(&p.mapOut, X_out, b.d / 8 * 8, a.T, (uint64_t)b.d * 2, 64, 32, true);
     p.mapA = p.mapB;
@@ -229,9 +239,13 @@ cudaError_t tc_decompress(const sn_basis &b, const TcArgs &a, __nv_bfloat16 *X_o
     p.ntiles = (int)((a.T + BM - 1) / BM);
     split_blocks(p.ntiles, p.nblk, sms, &p.bpi, &p.chunks);
     tile_order(a.T, a.seq_len, has_pe, p.has_pos, &p.reorder, &p.batches);
-    p.stages = expand_stages(a.gather, p.katoms, has_pe);
     const int grid = std::min(p.ntiles * p.chunks, sms);
-    return launch_expand(AMODE_REPACK, a.gather, p, grid, s);
+    if (a.gather) {
+        recon_stages(p.katoms, has_pe, &p.stages, &p.estages);
+        return launch_reconstruct(p, grid, s);
+    }
+    p.stages = expand_stages(false, p.katoms, 0);
+    return launch_expand(AMODE_REPACK, false, p, grid, s);
 }
 
 size_t tc_project_workspace(const sn_basis &b, int64_t cols)

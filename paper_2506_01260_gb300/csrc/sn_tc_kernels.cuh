@@ -90,7 +90,8 @@ struct ExpandParams {
     int k, katoms, kmma;
     int ncols, nblk, bpi, chunks, ntiles;
     int reorder, batches;
-    int stages;
+    int stages;          // B-operand stages
+    int estages;         // embedding stages (reconstruction)
 };
 
 struct ExpandPlan {
@@ -130,6 +131,36 @@ __host__ __device__ inline ExpandPlan expand_plan(bool gather, int katoms, int h
 __host__ __device__ constexpr int expand_threads(bool gather) { return gather ? 448 : 320; }
 constexpr int kExpandAcc = 4;     // TMEM accumulator buffers of expand_bn() columns
 
+// ---- reconstruction: out[r, n0:n0+128] = C[r, :] . U[n0:n0+128, :]^T + P rows + T_fixed rows
+// The A operand (the tile's C rows) lives in TMEM, double-buffered, next to three
+// fp32 accumulators, so shared memory holds only `sb` B stages of 128 U rows and
+// `se` embedding stages, each the [128 x 64] T_fixed tile and (with a positional
+// table) the [128 x 64] positional tile of one half of an output block.  The
+// epilogue writes each half's bf16 result over its T_fixed tile and stores it
+// from there, so no separate staging tile is needed.
+constexpr int kReconAcc = 3;              // accumulators of 128 columns
+constexpr uint32_t kReconACol = 384;      // first TMEM column of the A buffers
+constexpr uint32_t kReconAStride = 64;    // TMEM columns per A buffer (k <= 128)
+
+struct ReconPlan {
+    uint32_t b_bytes, t_bytes, e_bytes, bar_off, total;
+};
+
+__host__ __device__ inline ReconPlan recon_plan(int katoms, int has_pe, int sb, int se)
+{
+    ReconPlan p;
+    p.b_bytes = (uint32_t)katoms * BN_WIDE * 128;
+    p.t_bytes = kTile;
+    p.e_bytes = has_pe ? 2 * kTile : kTile;
+    p.bar_off = (uint32_t)sb * p.b_bytes + (uint32_t)se * p.e_bytes;
+    p.total = p.bar_off + 8 * (2 * sb + 3 * se + 2 * kReconAcc + 5) + 16 + 1024;
+    return p;
+}
+
+// warp 0 producer, warp 1 MMA, warps 2-5 and 6-9 two epilogue groups
+// (one per half block), warps 10-13 A operand and row gathers
+constexpr int kReconThreads = 448;
+
 // Row tile -> first row.  With `reorder`, tiles run position-block-major so the
 // b sequences of a batch that share positional rows are processed together
 // and the positional table is read from HBM once.
@@ -145,6 +176,7 @@ __host__ __device__ inline int64_t tile_row0(int tile, int reorder, int batches,
 // ---- host side -----------------------------------------------------------------------
 cudaError_t launch_contract(int mode, const ContractParams &p, int grid, cudaStream_t s);
 cudaError_t launch_expand(int amode, bool gather, const ExpandParams &p, int grid, cudaStream_t s);
+cudaError_t launch_reconstruct(const ExpandParams &p, int grid, cudaStream_t s);
 
 }  // namespace tc
 }  // namespace sn

@@ -1,0 +1,397 @@
+// sn_tc_reconstruct.cu — the forward reconstruction on the tcgen05 tensor cores,
+//
+//   X[t, :] = C[t, :] U^T + P[p_t, :] + T_fixed[id_t, :]          Sec. 4.3.1
+//
+// A work item is one 128-row tile and a run of 128-column output blocks.
+//   warp 0     TMA producer: per block, the 128 rows of U (the B operand,
+//              128-byte swizzled) into a ring of B stages;
+//   warp 1     TMEM allocation and tcgen05.mma into three fp32 accumulator
+//              buffers (M = 128, N = 128, K = k padded to 16) with the A
+//              operand read from TMEM; each commit frees the B stage and
+//              publishes the accumulator;
+//   warps 2-9  two epilogue groups, one per 64-column half of every block.  A
+//              thread drains its row of the group's half of the accumulator,
+//              adds the row's positional and T_fixed entries in fp32, rounds
+//              once to bf16 and writes the result over the T_fixed tile it just
+//              read; the warp then stores its 32 rows with one TMA store and
+//              frees the embedding stage once the store has read them;
+//   warps 10-13 write each item's C rows into one of two TMEM A buffers (a
+//              thread per row, zero-padded to a multiple of 16), then fill the
+//              ring of embedding stages: per half block, the T_fixed rows of
+//              the tile's ids (and the positional rows when positions are not
+//              one contiguous run) with 16-byte cp.async copies into swizzled
+//              positions, or the positional tile with one TMA load.  Each
+//              thread hands its copies to the stage's barrier
+//              (cp.async.mbarrier.arrive), which completes when all of them
+//              have landed, so the gather warps never wait for their own copies
+//              and every free stage can have copies in flight.
+// The embeddings never pass through the tensor core, so the MMA issues only the
+// k/16 instructions of C U^T per block; the B ring and the embedding ring are
+// separate, so U rows are released as soon as the MMAs have read them; with A
+// in TMEM, shared memory is left to the two rings.
+// Each CTA walks an item's blocks starting at its own offset, so the CTAs'
+// B-operand reads are spread over the L2 instead of converging on one slice.
+// Every wait is bounded (SN_EBIT_TIMEOUT); an aborting CTA drains its copies
+// and MMAs and frees TMEM before it returns.
+#include "sn_tc.cuh"
+#include "sn_tc_kernels.cuh"
+
+namespace sn {
+namespace tc {
+namespace {
+
+constexpr int NB = BN_WIDE;
+constexpr uint32_t kTmemCols = 512;
+static_assert(kReconAcc * NB <= (int)kReconACol && kReconACol + 2 * kReconAStride <= kTmemCols,
+              "TMEM plan");
+
+__device__ __forceinline__ int block_at(int blk0, int blk1, int j)
+{
+    const int nb = blk1 - blk0;
+    return blk0 + (int)((j + blockIdx.x) % nb);
+}
+
+// acc + P + T_fixed for two adjacent columns, rounded once to bf16
+__device__ __forceinline__ uint32_t add_emb(float a0, float a1, uint32_t pe, uint32_t te)
+{
+    return pack_bf16(a0 + bf_lo(pe) + bf_lo(te), a1 + bf_hi(pe) + bf_hi(te));
+}
+
+__global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_constant__ ExpandParams p)
+{
+    extern __shared__ uint8_t smem_raw[];
+    uint32_t base = smem_u32(smem_raw);
+    const uint32_t pad = (1024u - (base & 1023u)) & 1023u;
+    base += pad;
+    uint8_t *smem = smem_raw + pad;
+
+    const int SB = p.stages, SE = p.estages;
+    const ReconPlan pl = recon_plan(p.katoms, p.has_pe, SB, SE);
+    const uint32_t b0 = base, e0 = b0 + SB * pl.b_bytes;
+    const uint32_t bar = base + pl.bar_off;
+    const uint32_t bfull_b = bar, bempty_b = bar + 8 * SB;
+    const uint32_t efull_b = bar + 16 * SB, pfull_b = efull_b + 8 * SE, eempty_b = pfull_b + 8 * SE;
+    const uint32_t accf_b = eempty_b + 8 * SE, acce_b = accf_b + 8 * kReconAcc;
+    const uint32_t afull_b = acce_b + 8 * kReconAcc, aempty_b = afull_b + 16;
+    const uint32_t drain_b = aempty_b + 16;
+    uint32_t *tmem_slot = (uint32_t *)(smem + pl.bar_off + 8 * (2 * SB + 3 * SE + 2 * kReconAcc + 5));
+    volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < SB; ++s) {
+            mbar_init(bfull_b + 8 * s, 1);
+            mbar_init(bempty_b + 8 * s, 1);
+        }
+        for (int s = 0; s < SE; ++s) {
+            mbar_init(efull_b + 8 * s, 128);  // one (copy-tracking) arrival per gather thread
+            mbar_init(pfull_b + 8 * s, 1);    // positional tile (TMA) or a plain arrival
+            mbar_init(eempty_b + 8 * s, 4);   // the four warps of one epilogue group
+        }
+        for (int b = 0; b < kReconAcc; ++b) {
+            mbar_init(accf_b + 8 * b, 1);
+            mbar_init(acce_b + 8 * b, 8);     // both epilogue groups
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(afull_b + 8 * b, 4);    // the four gather warps
+            mbar_init(aempty_b + 8 * b, 1);
+        }
+        mbar_init(drain_b, 1);
+        *abort_flag = 0;
+        mbar_fence_init();
+    }
+    if (warp == 1)
+        tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    const int nitems = p.ntiles * p.chunks;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ B producer
+        if (lane == 0)
+            tma_prefetch(&p.mapB);
+        uint32_t g = 0;
+        bool ok = true;
+        for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x) {
+            const int ch = item % p.chunks;
+            const int blk0 = ch * p.bpi, blk1 = min(blk0 + p.bpi, p.nblk);
+            for (int j = 0; j < blk1 - blk0; ++j, ++g) {
+                const int blk = block_at(blk0, blk1, j);
+                const int s = g % SB;
+                if (!warp_wait(bempty_b + 8 * s, ((g / SB) & 1) ^ 1, abort_flag, p.err)) {
+                    ok = false;
+                    break;
+                }
+                if (lane == 0) {
+                    const uint32_t fb = bfull_b + 8 * s, st = b0 + s * pl.b_bytes;
+                    mbar_arrive_tx(fb, pl.b_bytes);
+                    for (int a = 0; a < p.katoms; ++a)
+                        tma_load_2d(st + a * (NB * 128), &p.mapB, a * 64, blk * NB, fb);
+                }
+                __syncwarp();
+            }
+        }
+        if (!ok && lane == 0)
+            for (uint32_t i = g > (uint32_t)SB ? g - SB : 0; i < g; ++i)
+                drain_wait(bfull_b + 8 * (i % SB), (i / SB) & 1);
+        __syncwarp();
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16(BM, NB);
+            uint32_t g = 0, it = 0;
+            bool ok = true;
+            for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++it) {
+                const int ch = item % p.chunks;
+                const int blk0 = ch * p.bpi, blk1 = min(blk0 + p.bpi, p.nblk);
+                const uint32_t ab = it & 1;
+                if (!mbar_wait(afull_b + 8 * ab, (it >> 1) & 1, abort_flag, p.err)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t a_tmem = tmem + kReconACol + ab * kReconAStride;
+                for (int j = 0; j < blk1 - blk0; ++j, ++g) {
+                    const int s = g % SB;
+                    const uint32_t b = g % kReconAcc;
+                    if (!mbar_wait(bfull_b + 8 * s, (g / SB) & 1, abort_flag, p.err) ||
+                        !mbar_wait(acce_b + 8 * b, ((g / kReconAcc) & 1) ^ 1, abort_flag, p.err)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t st = b0 + s * pl.b_bytes;
+                    const uint32_t d_tmem = tmem + b * NB;
+                    for (int kk = 0; kk < p.kmma; ++kk) {
+                        const uint32_t a = kk >> 2, off = (kk & 3) * 32;
+                        mma_bf16_ta(d_tmem, a_tmem + 8 * kk, sdesc_sw128(st + a * (NB * 128) + off),
+                                    idesc, kk > 0 ? 1u : 0u);
+                    }
+                    mma_commit(bempty_b + 8 * s);    // U rows free once these MMAs finish
+                    mma_commit(accf_b + 8 * b);
+                }
+                if (ok)
+                    mma_commit(aempty_b + 8 * ab);   // A buffer free once this item's MMAs finish
+            }
+            if (!ok) {
+                mma_commit(drain_b);
+                drain_wait(drain_b, 0);
+            }
+        }
+        __syncwarp();
+    } else if (warp < 10) {
+        // ------------------------------------------------------------ epilogue groups
+        const int q = warp & 3;
+        const int grp = (warp - 2) >> 2;     // the group's 64-column half of each block
+        const int row = 32 * q + lane;
+        uint32_t g = 0;
+        bool ok = true;
+        for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x) {
+            const int tile = item / p.chunks, ch = item % p.chunks;
+            const int blk0 = ch * p.bpi, blk1 = min(blk0 + p.bpi, p.nblk);
+            const int64_t r0 = tile_row0(tile, p.reorder, p.batches, p.seq_len);
+            bool bad = false;
+            {
+                const int64_t t = r0 + row;
+                if (t < p.rows) {
+                    const int id = p.ids[t];
+                    bad = id < 0 || id >= p.vocab;
+                    if (p.has_pe && p.has_pos) {
+                        const int ps = p.pos[t];
+                        bad = bad || ps < 0 || ps >= p.seq_len;
+                    }
+                    if (bad && ch == 0)
+                        atomicOr(p.err, SN_EBIT_BAD_ID);
+                }
+            }
+            for (int j = 0; j < blk1 - blk0 && ok; ++j, ++g) {
+                const int blk = block_at(blk0, blk1, j);
+                const uint32_t b = g % kReconAcc;
+                const uint32_t e = 2 * g + grp, es = e % SE, ph = (e / SE) & 1;
+                if (!warp_wait(accf_b + 8 * b, (g / kReconAcc) & 1, abort_flag, p.err)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                float v[64];
+                const uint32_t taddr = tmem + b * NB + 64 * grp + ((uint32_t)(32 * q) << 16);
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    tmem_ld16(taddr + 16 * i, *(float(*)[16])(v + 16 * i));
+                tmem_ld_wait();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0)
+                    mbar_arrive(acce_b + 8 * b);
+                if (!warp_wait(efull_b + 8 * es, ph, abort_flag, p.err) ||
+                    !warp_wait(pfull_b + 8 * es, ph, abort_flag, p.err)) {
+                    ok = false;
+                    break;
+                }
+                // the thread's own row of the T_fixed and positional tiles (a
+                // quarter-warp's 8 rows fall in 8 different banks), summed in
+                // fp32 and written back over the T_fixed tile
+                const uint32_t tb = e0 + es * pl.e_bytes;
+#pragma unroll
+                for (int cb = 0; cb < 8; cb += 4) {
+                    // all loads of four chunks first, then their sums
+                    uint4 tv[4], pv[4];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const uint32_t off = sw128(row, cb + i);
+                        tv[i] = lds128(tb + off);
+                        pv[i] = p.has_pe ? lds128(tb + pl.t_bytes + off) : make_uint4(0, 0, 0, 0);
+                    }
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const float *a = v + 8 * (cb + i);
+                        uint4 o = make_uint4(add_emb(a[0], a[1], pv[i].x, tv[i].x),
+                                             add_emb(a[2], a[3], pv[i].y, tv[i].y),
+                                             add_emb(a[4], a[5], pv[i].z, tv[i].z),
+                                             add_emb(a[6], a[7], pv[i].w, tv[i].w));
+                        if (bad)
+                            o = make_uint4(0, 0, 0, 0);
+                        sts128(tb + sw128(row, cb + i), o);
+                    }
+                }
+                // the warp's 32 rows leave with one TMA store (clipped at the
+                // tensor's edges); the stage is free once the store has read them
+                fence_async_smem();
+                __syncwarp();
+                {
+                    const int c0 = blk * NB + 64 * grp;
+                    if (lane == 0 && r0 + 32 * q < p.rows && c0 < p.ncols8) {
+                        tma_store_2d(&p.mapOut, tb + 32 * q * 128, c0, (int)(r0 + 32 * q));
+                        bulk_commit();
+                        bulk_wait_read0();
+                    }
+                }
+                __syncwarp();
+                if (lane == 0)
+                    mbar_arrive(eempty_b + 8 * es);
+            }
+        }
+        if (lane == 0)
+            bulk_wait_all0();
+    } else {
+        // ------------------------------------------------------------ embedding gathers
+        const int tt = threadIdx.x - 320;    // 0..127
+        const int arow = 32 * (warp & 3) + lane;   // this thread's TMEM lane (A row)
+        if (tt == 0 && p.has_pe)
+            tma_prefetch(&p.mapPE);
+        uint32_t g = 0, e = 0, it = 0;
+        bool ok = true;
+        for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++it) {
+            const int tile = item / p.chunks, ch = item % p.chunks;
+            const int blk0 = ch * p.bpi, blk1 = min(blk0 + p.bpi, p.nblk);
+            const int64_t r0 = tile_row0(tile, p.reorder, p.batches, p.seq_len);
+            {
+                // A operand: row arow of the tile's C rows, two bf16 per TMEM
+                // column, zero past k (and for rows past the end)
+                const uint32_t ab = it & 1;
+                if (!warp_wait(aempty_b + 8 * ab, ((it >> 1) & 1) ^ 1, abort_flag, p.err)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const int64_t t = r0 + arow;
+                const unsigned short *crow = (const unsigned short *)p.C + t * p.k;
+                const uint32_t a_tmem = tmem + ((uint32_t)(32 * (warp & 3)) << 16) + kReconACol +
+                                        ab * kReconAStride;
+                for (int w0 = 0; w0 < 8 * p.kmma; w0 += 16) {
+                    uint32_t h[16];
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        const int j0 = 2 * (w0 + i);
+                        const uint32_t lo = (t < p.rows && j0 < p.k) ? __ldg(crow + j0) : 0u;
+                        const uint32_t hi = (t < p.rows && j0 + 1 < p.k) ? __ldg(crow + j0 + 1) : 0u;
+                        h[i] = lo | (hi << 16);
+                    }
+                    tmem_st16(a_tmem + w0, h);
+                }
+                tmem_st_wait();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0)
+                    mbar_arrive(afull_b + 8 * ab);
+            }
+            const bool pe_tile = p.has_pe && !p.has_pos && (r0 % p.seq_len) + BM <= p.seq_len;
+            // element offsets of this thread's 8 rows in T_fixed and P (invalid
+            // ids / positions read row 0; the epilogue zeroes those rows)
+            int64_t trow[8], prow[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int64_t t = r0 + (tt >> 3) + 16 * u;
+                int64_t id = 0, ps = 0;
+                if (t < p.rows) {
+                    id = p.ids[t];
+                    if (id < 0 || id >= p.vocab)
+                        id = 0;
+                    if (p.has_pe) {
+                        ps = p.has_pos ? (int64_t)p.pos[t] : t % p.seq_len;
+                        if (ps < 0 || ps >= p.seq_len)
+                            ps = 0;
+                    }
+                }
+                trow[u] = id * p.ncols;
+                prow[u] = ps * p.ncols;
+            }
+            for (int j = 0; j < blk1 - blk0 && ok; ++j, ++g) {
+                const int blk = block_at(blk0, blk1, j);
+                for (int hh = 0; hh < 2; ++hh, ++e) {
+                    const uint32_t es = e % SE;
+                    if (!warp_wait(eempty_b + 8 * es, ((e / SE) & 1) ^ 1, abort_flag, p.err)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t tb = e0 + es * pl.e_bytes;
+                    const int col0 = blk * NB + 64 * hh;
+                    if (tt == 0) {
+                        const uint32_t pb = pfull_b + 8 * es;
+                        if (pe_tile) {
+                            mbar_arrive_tx(pb, kTile);
+                            tma_load_2d(tb + pl.t_bytes, &p.mapPE, col0, (int)(r0 % p.seq_len), pb);
+                        } else {
+                            mbar_arrive(pb);
+                        }
+                    }
+                    gather_tile_async(tb, p.tok, trow, col0, p.ncols, tt);
+                    if (p.has_pe && !pe_tile)
+                        gather_tile_async(tb + pl.t_bytes, p.pe, prow, col0, p.ncols, tt);
+                    cp_async_arrive(efull_b + 8 * es);
+                }
+            }
+        }
+        cp_async_wait0();
+        // positional tiles still in flight after an abort
+        if (!ok && tt == 0)
+            for (uint32_t i = e > (uint32_t)SE ? e - SE : 0; i < e; ++i)
+                drain_wait(pfull_b + 8 * (i % SE), (i / SE) & 1);
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_reconstruct(const ExpandParams &p, int grid, cudaStream_t s)
+{
+    const ReconPlan pl = recon_plan(p.katoms, p.has_pe, p.stages, p.estages);
+    cudaError_t e = cudaFuncSetAttribute(k_reconstruct, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         pl.total);
+    if (e != cudaSuccess)
+        return e;
+    k_reconstruct<<<grid, kReconThreads, pl.total, s>>>(p);
+    count_launch();
+    return cudaGetLastError();
+}
+
+}  // namespace tc
+}  // namespace sn
