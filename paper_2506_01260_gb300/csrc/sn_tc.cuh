@@ -1,5 +1,5 @@
 // sn_tc.cuh — inline-PTX building blocks for the sm_103a tensor-core kernels:
-// mbarriers with bounded waits, TMA tile / gather4 loads and tile stores,
+// mbarriers with bounded waits, TMA tile loads and stores, cp.async row gathers,
 // tcgen05 TMEM allocation, MMA (kind::f16, bf16 in, fp32 accumulate), commit
 // and TMEM loads, and the shared-memory matrix descriptors for the 128-byte
 // swizzled K-major operand layout.
@@ -45,12 +45,6 @@ __device__ __forceinline__ void mbar_arrive_tx(uint32_t bar, uint32_t bytes)
 {
     asm volatile("mbarrier.arrive.expect_tx.release.cta.shared::cta.b64 _, [%0], %1;" ::"r"(bar),
                  "r"(bytes)
-                 : "memory");
-}
-// Raise the expected transaction bytes of the current phase without arriving.
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes)
-{
-    asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(bytes)
                  : "memory");
 }
 __device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity)
@@ -139,17 +133,6 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *m, 
         "l"(m), "r"(x), "r"(y), "r"(bar)
         : "memory");
 }
-// Four rows r0..r3 of a 2-D tensor, columns x .. x+box-1, into four
-// consecutive box rows of shared memory (the map's box is one row high).
-__device__ __forceinline__ void tma_gather4(uint32_t dst, const CUtensorMap *m, int x, int r0,
-                                            int r1, int r2, int r3, uint32_t bar)
-{
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::"
-        "bytes [%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(dst),
-        "l"(m), "r"(x), "r"(r0), "r"(r1), "r"(r2), "r"(r3), "r"(bar)
-        : "memory");
-}
 __device__ __forceinline__ void tma_store_2d(const CUtensorMap *m, uint32_t src, int x, int y)
 {
     asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::
@@ -161,10 +144,6 @@ __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.comm
 __device__ __forceinline__ void bulk_wait_read0()
 {
     asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
-}
-__device__ __forceinline__ void bulk_wait_read1()
-{
-    asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
 }
 __device__ __forceinline__ void bulk_wait_all0()
 {
@@ -354,29 +333,7 @@ __device__ __forceinline__ void gather_tile_async(uint32_t dst, const __nv_bfloa
     }
 }
 
-// Rewrite a [128 x 128 B] tile of unswizzled rows (as tile::gather4 leaves
-// them) into the 128-byte swizzle layout the MMA reads, in place.  Called by
-// the 128 threads tt = 0..127 of four warps; every row is read and rewritten
-// by one quarter-warp, so only warp-level ordering is needed.
-__device__ __forceinline__ void swizzle_rows_in_place(uint32_t tile, int tt)
-{
-    uint4 v[8];
-#pragma unroll
-    for (int u = 0; u < 8; ++u)
-        v[u] = lds128(tile + (uint32_t)(tt + 128 * u) * 16);
-    __syncwarp();
-#pragma unroll
-    for (int u = 0; u < 8; ++u) {
-        const int unit = tt + 128 * u, r = unit >> 3, c = unit & 7;
-        if (r & 7)
-            sts128(tile + sw128(r, c), v[u]);
-    }
-}
 
-__device__ __forceinline__ void named_bar_sync(int id, int nthreads)
-{
-    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
-}
 
 }  // namespace tc
 }  // namespace sn

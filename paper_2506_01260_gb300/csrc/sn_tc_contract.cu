@@ -19,7 +19,10 @@
 //              fp32 partial rows);
 //   warps 6-9  CMODE_X: gather the T_fixed rows (and non-contiguous positional
 //              rows) with 16-byte cp.async copies straight into their swizzled
-//              positions, then fence toward the async proxy and arrive.
+//              positions; each thread hands its copies to the stage's barrier
+//              (cp.async.mbarrier.arrive), so the gather warps never wait for
+//              their own copies, and the MMA thread fences toward the async
+//              proxy after the barrier completes.
 // Each CTA walks an item's chunks starting at its own offset, so the CTAs' U^T
 // reads are spread over the L2 instead of converging on one slice.
 // Every wait is bounded; a wait that expires raises SN_EBIT_TIMEOUT and the
@@ -60,7 +63,7 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
-            mbar_init(full_b + 8 * s, MODE == CMODE_X ? 1 + 4 : 1);
+            mbar_init(full_b + 8 * s, MODE == CMODE_X ? 1 + 128 : 1);   // TMA + gather threads
             mbar_init(rr_b + 8 * s, 4);
             mbar_init(empty_b + 8 * s, 1);
         }
@@ -158,6 +161,8 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
                         break;
                     }
                     tc_fence_after();
+                    if (MODE == CMODE_X)   // gathered rows (generic proxy) -> MMA reads
+                        fence_async_smem();
                     const uint32_t st = base + s * pl.stage_bytes;
                     const uint32_t ub = st + pl.a_bytes;
 #pragma unroll
@@ -307,7 +312,6 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
         // ------------------------------------------------------------ gather warps
         const int tt = threadIdx.x - 192;    // 0..127
         uint32_t g = 0;
-        int pend_s = -1;                     // stage whose copies are not yet signalled
         bool ok = true;
         for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x) {
             const int tile = item / p.splits, split = item % p.splits;
@@ -347,22 +351,10 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
                 gather_tile_async(tb, p.tok, trow, (int64_t)kc * BK, p.d, tt);
                 if (p.has_pe && !pe_tile)
                     gather_tile_async(tb + pl.raw_bytes, p.pe, prow, (int64_t)kc * BK, p.d, tt);
-                cp_async_commit();
-                if (pend_s >= 0) {   // the previous stage's copies have landed
-                    cp_async_wait1();
-                    fence_async_smem();
-                    __syncwarp();
-                    if (lane == 0)
-                        mbar_arrive(full_b + 8 * pend_s);
-                }
-                pend_s = s;
+                cp_async_arrive(full_b + 8 * s);
             }
         }
         cp_async_wait0();
-        fence_async_smem();
-        __syncwarp();
-        if (pend_s >= 0 && lane == 0)
-            mbar_arrive(full_b + 8 * pend_s);
     }
 
     tc_fence_before();

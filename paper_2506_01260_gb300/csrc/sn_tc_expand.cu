@@ -1,31 +1,25 @@
-// sn_tc_expand.cu — the k -> d expansion on the tcgen05 tensor cores.
+// sn_tc_expand.cu — the plain k -> d expansion on the tcgen05 tensor cores.
 //
-//   decompress_fwd  X[t, :] = C[t, :] U^T + P[p_t, :] + T_fixed[id_t, :]   Sec. 4.3.1
 //   decompress_bwd  G[t, :] = C[t, :] U^T                                 Sec. 4.4
 //   project (b)     W'[i, :] = U[i, :] A   with A = U^T W from the first pass
 //
-// A work item is one 128-row tile and a run of NB-column output blocks (NB = 64
-// for the reconstruction, 128 otherwise).
-//   warp 0     TMA producer: per block, the NB rows of the B operand (U, or
-//              A^T) and, for the reconstruction with contiguous positions, the
-//              positional tile; per item, the A operand when it comes from a
-//              tensor map (all 128-byte swizzled);
+// (The forward reconstruction, which also adds the embeddings, has its own
+// kernel.)  A work item is one 128-row tile and a run of 128-column output
+// blocks.
+//   warp 0     TMA producer: per block, the 128 rows of the B operand (U, or
+//              A^T); per item, the A operand when it comes from a tensor map
+//              (all 128-byte swizzled);
 //   warp 1     TMEM allocation and tcgen05.mma into four fp32 accumulator
-//              buffers (M = 128, N = NB): C U^T over K = k padded to 16,
-//              then, for the reconstruction, + T_fixed rows . I + P rows . I
-//              with a resident 64 x 64 identity operand, so the embeddings are
-//              added in fp32 inside the tensor core;
+//              buffers (M = 128, N = 128): C U^T over K = k padded to 16;
 //   warps 2-9  two epilogue groups taking alternate blocks: drain the
-//              accumulator, round once to bf16 into the group's swizzled
-//              staging tile and write each warp's 32 rows with coalesced
-//              16-byte stores (the TMA unit is left to the loads); together the
-//              groups repack each item's C rows into the swizzled K-major A
-//              operand (zero-padded).  Stages are released by the MMA commit.
+//              accumulator 64 columns at a time, round once to bf16 into the
+//              group's swizzled staging tile and write each warp's 32 rows with
+//              coalesced 16-byte stores (the TMA unit is left to the loads);
+//              together the groups repack each item's C rows into the swizzled
+//              K-major A operand (zero-padded).  Stages are released by the MMA
+//              commit.
 // Each CTA walks an item's blocks starting at its own offset, so the CTAs'
-// B-operand reads are spread over the L2 instead of converging on one slice;
-//   warps 10-13 (reconstruction only) build the identity, then gather each
-//              block's T_fixed rows (and non-contiguous positional rows) with
-//              16-byte cp.async copies straight into their swizzled positions.
+// B-operand reads are spread over the L2 instead of converging on one slice.
 // Every wait is bounded (SN_EBIT_TIMEOUT); an aborting CTA drains its copies
 // and MMAs and frees TMEM before it returns.
 #include "sn_tc.cuh"
@@ -43,9 +37,8 @@ __device__ __forceinline__ int block_at(int blk0, int blk1, int j)
     return blk0 + (int)((j + blockIdx.x) % nb);
 }
 
-template <int AMODE, bool GATHER>
-__global__ void __launch_bounds__(expand_threads(GATHER), 1)
-    k_expand(const __grid_constant__ ExpandParams p)
+template <int AMODE>
+__global__ void __launch_bounds__(kExpandThreads, 1) k_expand(const __grid_constant__ ExpandParams p)
 {
     extern __shared__ uint8_t smem_raw[];
     uint32_t base = smem_u32(smem_raw);
@@ -54,24 +47,23 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
     uint8_t *smem = smem_raw + pad;
 
     const int S = p.stages;
-    const ExpandPlan pl = expand_plan(GATHER, p.katoms, p.has_pe, S);
-    const uint32_t a_s = base, id_s = base + pl.a_bytes, out_s = id_s + pl.id_bytes;
+    const ExpandPlan pl = expand_plan(p.katoms, S);
+    const uint32_t a_s = base, out_s = base + pl.a_bytes;
     const uint32_t stage0 = out_s + pl.out_bytes;
     const uint32_t bar = base + pl.bar_off;
     const uint32_t full_b = bar, empty_b = bar + 8 * S;
-    const uint32_t accf_b = bar + 24 * S, acce_b = accf_b + 8 * kExpandAcc;
+    const uint32_t accf_b = bar + 16 * S, acce_b = accf_b + 8 * kExpandAcc;
     const uint32_t afull_b = acce_b + 8 * kExpandAcc, aempty_b = afull_b + 8;
-    const uint32_t drain_b = aempty_b + 8, idready_b = drain_b + 8;
-    uint32_t *tmem_slot = (uint32_t *)(smem + pl.bar_off + 8 * (3 * S + 12));
+    const uint32_t drain_b = aempty_b + 8;
+    uint32_t *tmem_slot = (uint32_t *)(smem + pl.bar_off + 8 * (2 * S + 2 * kExpandAcc + 3));
     volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    constexpr int NB = expand_bn(GATHER);
-    static_assert(!GATHER || NB == BN, "the gathered rows and the identity are 64 wide");
+    constexpr int NB = BN_WIDE;
     constexpr uint32_t kTmemCols = kExpandAcc * NB;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
-            mbar_init(full_b + 8 * s, GATHER ? 1 + 4 : 1);
+            mbar_init(full_b + 8 * s, 1);
             mbar_init(empty_b + 8 * s, 1);
         }
         for (int b = 0; b < kExpandAcc; ++b) {
@@ -81,7 +73,6 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
         mbar_init(afull_b, AMODE == AMODE_REPACK ? 8 : 1);
         mbar_init(aempty_b, 1);
         mbar_init(drain_b, 1);
-        mbar_init(idready_b, 4);
         *abort_flag = 0;
         mbar_fence_init();
     }
@@ -99,8 +90,6 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
             tma_prefetch(&p.mapB);
             if (AMODE == AMODE_TMA)
                 tma_prefetch(&p.mapA);
-            if (GATHER && p.has_pe)
-                tma_prefetch(&p.mapPE);
         }
         uint32_t g = 0, it = 0;
         bool ok = true;
@@ -120,9 +109,7 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                 }
                 __syncwarp();
             }
-            const bool pe_tile =
-                GATHER && p.has_pe && !p.has_pos && (r0 % p.seq_len) + BM <= p.seq_len;
-            const uint32_t tx = pl.b_bytes + (pe_tile ? kTile : 0);
+            const uint32_t tx = pl.b_bytes;
             for (int j = 0; j < blk1 - blk0; ++j, ++g) {
                 const int blk = block_at(blk0, blk1, j);
                 const int s = g % S;
@@ -137,9 +124,6 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                     mbar_arrive_tx(fb, tx);
                     for (int a = 0; a < p.katoms; ++a)
                         tma_load_2d(st + a * (NB * 128), &p.mapB, a * 64, blk * NB, fb);
-                    if (pe_tile)
-                        tma_load_2d(st + pl.b_bytes + pl.t_bytes, &p.mapPE, blk * BN,
-                                    (int)(r0 % p.seq_len), fb);
                 }
                 __syncwarp();
             }
@@ -157,8 +141,6 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
             const uint32_t idesc = idesc_bf16(BM, NB);
             uint32_t g = 0, it = 0;
             bool ok = true;
-            if (GATHER && !mbar_wait(idready_b, 0, abort_flag, p.err))
-                ok = false;
             for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++it) {
                 const int ch = item % p.chunks;
                 const int blk0 = ch * p.bpi, blk1 = min(blk0 + p.bpi, p.nblk);
@@ -182,17 +164,6 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                         const uint32_t a = kk >> 2, off = (kk & 3) * 32;
                         mma_bf16(d_tmem, sdesc_sw128(a_s + a * kTile + off),
                                  sdesc_sw128(st + a * (NB * 128) + off), idesc, kk > 0 ? 1u : 0u);
-                    }
-                    if (GATHER) {   // + T_fixed rows . I + P rows . I
-                        const uint32_t tb = st + pl.b_bytes;
-#pragma unroll
-                        for (int kk = 0; kk < BN / 16; ++kk) {
-                            const uint64_t idd = sdesc_sw128(id_s + kk * 32);
-                            mma_bf16(d_tmem, sdesc_sw128(tb + kk * 32), idd, idesc, 1u);
-                            if (p.has_pe)
-                                mma_bf16(d_tmem, sdesc_sw128(tb + pl.t_bytes + kk * 32), idd,
-                                         idesc, 1u);
-                        }
                     }
                     mma_commit(empty_b + 8 * s);     // stage free once these MMAs finish
                     mma_commit(accf_b + 8 * b);
@@ -255,20 +226,6 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                 if (lane == 0)
                     mbar_arrive(afull_b);
             }
-            bool bad = false;
-            if (GATHER) {
-                const int64_t t = r0 + row;
-                if (t < p.rows) {
-                    const int id = p.ids[t];
-                    bad = id < 0 || id >= p.vocab;
-                    if (p.has_pe && p.has_pos) {
-                        const int ps = p.pos[t];
-                        bad = bad || ps < 0 || ps >= p.seq_len;
-                    }
-                    if (bad && ch == 0)
-                        atomicOr(p.err, SN_EBIT_BAD_ID);
-                }
-            }
             for (int j = 0; j < blk1 - blk0; ++j, ++g) {
                 if ((int)(g & 1) != grp)
                     continue;
@@ -300,17 +257,15 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
                     }
 #pragma unroll
                     for (int c = 0; c < 8; ++c) {
-                        uint4 o = make_uint4(pack_bf16(v[8 * c + 0], v[8 * c + 1]),
-                                             pack_bf16(v[8 * c + 2], v[8 * c + 3]),
-                                             pack_bf16(v[8 * c + 4], v[8 * c + 5]),
-                                             pack_bf16(v[8 * c + 6], v[8 * c + 7]));
-                        if (bad)
-                            o = make_uint4(0, 0, 0, 0);
-                        sts128(slot + h * kTile + sw128(row, c), o);
+                        sts128(slot + h * kTile + sw128(row, c),
+                               make_uint4(pack_bf16(v[8 * c + 0], v[8 * c + 1]),
+                                          pack_bf16(v[8 * c + 2], v[8 * c + 3]),
+                                          pack_bf16(v[8 * c + 4], v[8 * c + 5]),
+                                          pack_bf16(v[8 * c + 6], v[8 * c + 7])));
                     }
                     // columns past the 8-aligned width are written element by element
                     const int ch0 = c0 + 64 * h;
-                    if (!GATHER && ch0 + 64 > p.ncols8 && p.ncols > p.ncols8) {
+                    if (ch0 + 64 > p.ncols8 && p.ncols > p.ncols8) {
                         const int64_t t = r0 + row;
                         if (t < p.rows) {
 #pragma unroll
@@ -338,79 +293,6 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
             }
         }
 
-    } else if (GATHER) {
-        // ------------------------------------------------------------ gather warps
-        const int tt = threadIdx.x - 320;    // 0..127
-        // identity B operand: 64 rows (N) x 64 columns (K), swizzled
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            const int unit = tt + 128 * u, n = unit >> 3, c = unit & 7;
-            // row n holds bf16 1.0 at column n: chunk n / 8, element n % 8
-            const uint32_t one = (n & 1) ? 0x3F800000u : 0x00003F80u;
-            const int word = ((n >> 3) == c) ? ((n & 7) >> 1) : -1;
-            sts128(id_s + sw128(n, c), make_uint4(word == 0 ? one : 0u, word == 1 ? one : 0u,
-                                                  word == 2 ? one : 0u, word == 3 ? one : 0u));
-        }
-        fence_async_smem();
-        __syncwarp();
-        if (lane == 0)
-            mbar_arrive(idready_b);
-        uint32_t g = 0;
-        int pend_s = -1;                     // stage whose copies are not yet signalled
-        bool ok = true;
-        for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x) {
-            const int tile = item / p.chunks, ch = item % p.chunks;
-            const int blk0 = ch * p.bpi, blk1 = min(blk0 + p.bpi, p.nblk);
-            const int64_t r0 = tile_row0(tile, p.reorder, p.batches, p.seq_len);
-            const bool pe_tile = p.has_pe && !p.has_pos && (r0 % p.seq_len) + BM <= p.seq_len;
-            // element offsets of this thread's 8 rows in T_fixed and P (invalid
-            // ids / positions read row 0; the epilogue zeroes those rows)
-            int64_t trow[8], prow[8];
-#pragma unroll
-            for (int u = 0; u < 8; ++u) {
-                const int64_t t = r0 + (tt >> 3) + 16 * u;
-                int64_t id = 0, ps = 0;
-                if (t < p.rows) {
-                    id = p.ids[t];
-                    if (id < 0 || id >= p.vocab)
-                        id = 0;
-                    if (p.has_pe) {
-                        ps = p.has_pos ? (int64_t)p.pos[t] : t % p.seq_len;
-                        if (ps < 0 || ps >= p.seq_len)
-                            ps = 0;
-                    }
-                }
-                trow[u] = id * p.ncols;
-                prow[u] = ps * p.ncols;
-            }
-            for (int j = 0; j < blk1 - blk0; ++j, ++g) {
-                const int blk = block_at(blk0, blk1, j);
-                const int s = g % S;
-                const uint32_t n = g / S;
-                if (!warp_wait(empty_b + 8 * s, (n & 1) ^ 1, abort_flag, p.err)) {
-                    ok = false;
-                    break;
-                }
-                const uint32_t tb = stage0 + s * pl.stage_bytes + pl.b_bytes;
-                gather_tile_async(tb, p.tok, trow, (int64_t)blk * BN, p.ncols, tt);
-                if (p.has_pe && !pe_tile)
-                    gather_tile_async(tb + pl.t_bytes, p.pe, prow, (int64_t)blk * BN, p.ncols, tt);
-                cp_async_commit();
-                if (pend_s >= 0) {   // the previous stage's copies have landed
-                    cp_async_wait1();
-                    fence_async_smem();
-                    __syncwarp();
-                    if (lane == 0)
-                        mbar_arrive(full_b + 8 * pend_s);
-                }
-                pend_s = s;
-            }
-        }
-        cp_async_wait0();
-        fence_async_smem();
-        __syncwarp();
-        if (pend_s >= 0 && lane == 0)
-            mbar_arrive(full_b + 8 * pend_s);
     }
 
     tc_fence_before();
@@ -423,26 +305,20 @@ __global__ void __launch_bounds__(expand_threads(GATHER), 1)
 
 }  // namespace
 
-cudaError_t launch_expand(int amode, bool gather, const ExpandParams &p, int grid, cudaStream_t s)
+cudaError_t launch_expand(int amode, const ExpandParams &p, int grid, cudaStream_t s)
 {
-    const ExpandPlan pl = expand_plan(gather, p.katoms, p.has_pe, p.stages);
-    const int threads = expand_threads(gather);
+    const ExpandPlan pl = expand_plan(p.katoms, p.stages);
     cudaError_t e;
-    if (amode == AMODE_REPACK && gather) {
-        e = cudaFuncSetAttribute(k_expand<AMODE_REPACK, true>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, pl.total);
+    if (amode == AMODE_REPACK) {
+        e = cudaFuncSetAttribute(k_expand<AMODE_REPACK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 pl.total);
         if (e == cudaSuccess)
-            k_expand<AMODE_REPACK, true><<<grid, threads, pl.total, s>>>(p);
-    } else if (amode == AMODE_REPACK) {
-        e = cudaFuncSetAttribute(k_expand<AMODE_REPACK, false>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, pl.total);
-        if (e == cudaSuccess)
-            k_expand<AMODE_REPACK, false><<<grid, threads, pl.total, s>>>(p);
+            k_expand<AMODE_REPACK><<<grid, kExpandThreads, pl.total, s>>>(p);
     } else {
-        e = cudaFuncSetAttribute(k_expand<AMODE_TMA, false>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, pl.total);
+        e = cudaFuncSetAttribute(k_expand<AMODE_TMA>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 pl.total);
         if (e == cudaSuccess)
-            k_expand<AMODE_TMA, false><<<grid, threads, pl.total, s>>>(p);
+            k_expand<AMODE_TMA><<<grid, kExpandThreads, pl.total, s>>>(p);
     }
     if (e != cudaSuccess)
         return e;

@@ -80,10 +80,10 @@ int contract_stages(int mode, int n_pad, int k, int has_pe)
     return s;
 }
 
-int expand_stages(bool gather, int katoms, int has_pe)
+int expand_stages(int katoms)
 {
     int s = 8;
-    while (s > 2 && expand_plan(gather, katoms, has_pe, s).total > kSmemLimit)
+    while (s > 2 && expand_plan(katoms, s).total > kSmemLimit)
         --s;
     return s;
 }
@@ -244,8 +244,8 @@ cudaError_t tc_decompress(const sn_basis &b, const TcArgs &a, __nv_bfloat16 *X_o
         recon_stages(p.katoms, has_pe, &p.stages, &p.estages);
         return launch_reconstruct(p, grid, s);
     }
-    p.stages = expand_stages(false, p.katoms, 0);
-    return launch_expand(AMODE_REPACK, false, p, grid, s);
+    p.stages = expand_stages(p.katoms);
+    return launch_expand(AMODE_REPACK, p, grid, s);
 }
 
 size_t tc_project_workspace(const sn_basis &b, int64_t cols)
@@ -321,8 +321,8 @@ cudaError_t tc_project(const sn_basis &b, const __nv_bfloat16 *W, int64_t cols, 
     q.nblk = (int)((cols + BN_WIDE - 1) / BN_WIDE);
     q.ntiles = (b.d + BM - 1) / BM;
     split_blocks(q.ntiles, q.nblk, sms, &q.bpi, &q.chunks);
-    q.stages = expand_stages(false, q.katoms, 0);
-    return launch_expand(AMODE_TMA, false, q, std::min(q.ntiles * q.chunks, sms), s);
+    q.stages = expand_stages(q.katoms);
+    return launch_expand(AMODE_TMA, q, std::min(q.ntiles * q.chunks, sms), s);
 }
 
 }  // namespace sn

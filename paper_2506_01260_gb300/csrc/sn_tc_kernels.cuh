@@ -12,8 +12,7 @@ namespace tc {
 
 constexpr int BM = 128;          // rows (tokens / W columns / d rows) per tile = MMA M
 constexpr int BK = 64;           // contraction chunk: one 128-byte swizzle row of bf16
-constexpr int BN = 64;           // output columns per block of the reconstruction
-constexpr int BN_WIDE = 128;     // output columns per block of the plain expansion
+constexpr int BN_WIDE = 128;     // output columns per block of the expansions
 constexpr uint32_t kSmemLimit = 232448;   // 227 KB per CTA
 constexpr uint32_t kTile = BM * 128;      // one [128 x 64] bf16 swizzled tile
 
@@ -67,12 +66,13 @@ __host__ __device__ inline ContractPlan contract_plan(int mode, int n_pad, int k
     return p;
 }
 
-// ---- expansion: out[r, n0:n0+64] = A[r, :] . B[n0:n0+64, :]^T (+ gathered rows) ------
+// ---- expansion: out[r, n0:n0+128] = A[r, :] . B[n0:n0+128, :]^T ----------------------
 enum { AMODE_REPACK = 0, AMODE_TMA = 1 };
 
+// Shared by the plain expansion and the reconstruction.
 struct ExpandParams {
     CUtensorMap mapA;    // A by TMA: U padded [d, k64] (SW128, box 64 x 128)
-    CUtensorMap mapB;    // B rows: U padded [d, k64] | A^T [m, k64] (SW128, box 64 x NB)
+    CUtensorMap mapB;    // B rows: U padded [d, k64] | A^T [m, k64] (SW128, box 64 x 128)
     CUtensorMap mapOut;  // output [rows, ncols] (SW128, box 64 x 32)
     CUtensorMap mapPE;   // P (SW128, box 64 x 128), contiguous positions
     const __nv_bfloat16 *tok;   // T_fixed [vocab, ncols], rows gathered with cp.async
@@ -94,42 +94,29 @@ struct ExpandParams {
     int estages;         // embedding stages (reconstruction)
 };
 
+// warp 0 producer, warp 1 MMA, warps 2-5 and 6-9 two epilogue groups
+// (alternate blocks)
+constexpr int kExpandThreads = 320;
+constexpr int kExpandAcc = 4;     // TMEM accumulator buffers of 128 columns
+
 struct ExpandPlan {
-    uint32_t a_bytes, id_bytes, out_bytes, b_bytes, t_bytes, pe_bytes, stage_bytes, bar_off,
-        total;
+    uint32_t a_bytes, out_bytes, b_bytes, stage_bytes, bar_off, total;
 };
 
-// Output columns per block (the MMA's N): the reconstruction keeps 64 so that a
-// stage still holds the gathered T_fixed and positional rows; the plain
-// expansion takes 128, which halves the MMA instructions and per-block
-// hand-offs and reads each A slice from shared memory once per 128 columns.
-__host__ __device__ constexpr int expand_bn(bool gather) { return gather ? BN : BN_WIDE; }
-
-// Shared memory of the expansion: A operand | identity (gather) | two output
-// staging tiles | stages of [B rows | T_fixed rows | positional rows] | barriers.
-// A stage is released by the MMA commit; outputs have their own ring, so the
-// stores never hold back the loads.
-__host__ __device__ inline ExpandPlan expand_plan(bool gather, int katoms, int has_pe,
-                                                  int stages)
+// Shared memory of the plain expansion: A operand | two output staging tiles |
+// stages of B rows | barriers.  A stage is released by the MMA commit; outputs
+// have their own staging, so the stores never hold back the loads.
+__host__ __device__ inline ExpandPlan expand_plan(int katoms, int stages)
 {
     ExpandPlan p;
-    const uint32_t nb = (uint32_t)expand_bn(gather);
     p.a_bytes = (uint32_t)katoms * kTile;
-    p.id_bytes = gather ? BN * 128 : 0;           // 64 x 64 bf16 identity, swizzled
-    p.out_bytes = 2 * BM * nb * 2;                // one staging tile per epilogue group
-    p.b_bytes = (uint32_t)katoms * nb * 128;
-    p.t_bytes = gather ? kTile : 0;
-    p.pe_bytes = (gather && has_pe) ? kTile : 0;
-    p.stage_bytes = p.b_bytes + p.t_bytes + p.pe_bytes;
-    p.bar_off = p.a_bytes + p.id_bytes + p.out_bytes + (uint32_t)stages * p.stage_bytes;
-    p.total = p.bar_off + 8 * (3 * stages + 12) + 16 + 1024;
+    p.out_bytes = 2 * BM * BN_WIDE * 2;           // one staging tile per epilogue group
+    p.b_bytes = (uint32_t)katoms * BN_WIDE * 128;
+    p.stage_bytes = p.b_bytes;
+    p.bar_off = p.a_bytes + p.out_bytes + (uint32_t)stages * p.stage_bytes;
+    p.total = p.bar_off + 8 * (2 * stages + 2 * kExpandAcc + 3) + 16 + 1024;
     return p;
 }
-
-// warp 0 producer, warp 1 MMA, warps 2-5 and 6-9 two epilogue groups
-// (alternate blocks), warps 10-13 row gathers (reconstruction only)
-__host__ __device__ constexpr int expand_threads(bool gather) { return gather ? 448 : 320; }
-constexpr int kExpandAcc = 4;     // TMEM accumulator buffers of expand_bn() columns
 
 // ---- reconstruction: out[r, n0:n0+128] = C[r, :] . U[n0:n0+128, :]^T + P rows + T_fixed rows
 // The A operand (the tile's C rows) lives in TMEM, double-buffered, next to three
@@ -175,7 +162,7 @@ __host__ __device__ inline int64_t tile_row0(int tile, int reorder, int batches,
 
 // ---- host side -----------------------------------------------------------------------
 cudaError_t launch_contract(int mode, const ContractParams &p, int grid, cudaStream_t s);
-cudaError_t launch_expand(int amode, bool gather, const ExpandParams &p, int grid, cudaStream_t s);
+cudaError_t launch_expand(int amode, const ExpandParams &p, int grid, cudaStream_t s);
 cudaError_t launch_reconstruct(const ExpandParams &p, int grid, cudaStream_t s);
 
 }  // namespace tc
