@@ -111,6 +111,17 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
     return ok != 0;
 }
 
+// Bounded wait executed by all 32 lanes together: every lane tests the barrier
+// itself (so each observes the completed phase with acquire semantics) and the
+// lanes agree on the outcome.  All 32 lanes must call it.
+__device__ __forceinline__ bool warp_wait_all(uint32_t bar, uint32_t parity, volatile int *abort,
+                                              unsigned int *err)
+{
+    if (__all_sync(0xffffffffu, mbar_test(bar, parity)))
+        return true;
+    return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort, err));
+}
+
 // Short bounded wait used only while draining after an abort.
 __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity)
 {
@@ -286,6 +297,24 @@ __device__ __forceinline__ void sts128(uint32_t a, uint4 v)
 __device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 // Two fp32 values -> packed bf16x2 (round-to-nearest-even), `lo` in the low half.
+// c + (bf16 in the low / high half of w), one fp32 rounding, no unpacking
+__device__ __forceinline__ float add_bf16_lo(uint32_t w, float c)
+{
+    float r;
+    asm("{ .reg .b16 l, h; mov.b32 {l, h}, %1; add.rn.f32.bf16 %0, l, %2; }"
+        : "=f"(r)
+        : "r"(w), "f"(c));
+    return r;
+}
+__device__ __forceinline__ float add_bf16_hi(uint32_t w, float c)
+{
+    float r;
+    asm("{ .reg .b16 l, h; mov.b32 {l, h}, %1; add.rn.f32.bf16 %0, h, %2; }"
+        : "=f"(r)
+        : "r"(w), "f"(c));
+    return r;
+}
+
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
 {
     uint32_t r;

@@ -140,7 +140,7 @@ __host__ __device__ inline ReconPlan recon_plan(int katoms, int has_pe, int sb, 
     p.t_bytes = kTile;
     p.e_bytes = has_pe ? 2 * kTile : kTile;
     p.bar_off = (uint32_t)sb * p.b_bytes + (uint32_t)se * p.e_bytes;
-    p.total = p.bar_off + 8 * (2 * sb + 3 * se + 2 * kReconAcc + 5) + 16 + 1024;
+    p.total = p.bar_off + 8 * (2 * sb + 2 * se + 2 * kReconAcc + 5) + 16 + 1024;
     return p;
 }
 

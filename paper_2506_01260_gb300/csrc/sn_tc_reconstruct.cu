@@ -54,7 +54,7 @@ __device__ __forceinline__ int block_at(int blk0, int blk1, int j)
 // acc + P + T_fixed for two adjacent columns, rounded once to bf16
 __device__ __forceinline__ uint32_t add_emb(float a0, float a1, uint32_t pe, uint32_t te)
 {
-    return pack_bf16(a0 + bf_lo(pe) + bf_lo(te), a1 + bf_hi(pe) + bf_hi(te));
+    return pack_bf16(add_bf16_lo(te, add_bf16_lo(pe, a0)), add_bf16_hi(te, add_bf16_hi(pe, a1)));
 }
 
 __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_constant__ ExpandParams p)
@@ -70,11 +70,11 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
     const uint32_t b0 = base, e0 = b0 + SB * pl.b_bytes;
     const uint32_t bar = base + pl.bar_off;
     const uint32_t bfull_b = bar, bempty_b = bar + 8 * SB;
-    const uint32_t efull_b = bar + 16 * SB, pfull_b = efull_b + 8 * SE, eempty_b = pfull_b + 8 * SE;
+    const uint32_t efull_b = bar + 16 * SB, eempty_b = efull_b + 8 * SE;
     const uint32_t accf_b = eempty_b + 8 * SE, acce_b = accf_b + 8 * kReconAcc;
     const uint32_t afull_b = acce_b + 8 * kReconAcc, aempty_b = afull_b + 16;
     const uint32_t drain_b = aempty_b + 16;
-    uint32_t *tmem_slot = (uint32_t *)(smem + pl.bar_off + 8 * (2 * SB + 3 * SE + 2 * kReconAcc + 5));
+    uint32_t *tmem_slot = (uint32_t *)(smem + pl.bar_off + 8 * (2 * SB + 2 * SE + 2 * kReconAcc + 5));
     volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -84,8 +84,9 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
             mbar_init(bempty_b + 8 * s, 1);
         }
         for (int s = 0; s < SE; ++s) {
-            mbar_init(efull_b + 8 * s, 128);  // one (copy-tracking) arrival per gather thread
-            mbar_init(pfull_b + 8 * s, 1);    // positional tile (TMA) or a plain arrival
+            // one copy-tracking arrival per gather thread + one for the
+            // positional tile (a TMA load, or a plain arrival without one)
+            mbar_init(efull_b + 8 * s, 128 + 1);
             mbar_init(eempty_b + 8 * s, 4);   // the four warps of one epilogue group
         }
         for (int b = 0; b < kReconAcc; ++b) {
@@ -210,7 +211,7 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
                 const int blk = block_at(blk0, blk1, j);
                 const uint32_t b = g % kReconAcc;
                 const uint32_t e = 2 * g + grp, es = e % SE, ph = (e / SE) & 1;
-                if (!warp_wait(accf_b + 8 * b, (g / kReconAcc) & 1, abort_flag, p.err)) {
+                if (!warp_wait_all(accf_b + 8 * b, (g / kReconAcc) & 1, abort_flag, p.err)) {
                     ok = false;
                     break;
                 }
@@ -225,8 +226,7 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
                 __syncwarp();
                 if (lane == 0)
                     mbar_arrive(acce_b + 8 * b);
-                if (!warp_wait(efull_b + 8 * es, ph, abort_flag, p.err) ||
-                    !warp_wait(pfull_b + 8 * es, ph, abort_flag, p.err)) {
+                if (!warp_wait_all(efull_b + 8 * es, ph, abort_flag, p.err)) {
                     ok = false;
                     break;
                 }
@@ -349,7 +349,7 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
                     const uint32_t tb = e0 + es * pl.e_bytes;
                     const int col0 = blk * NB + 64 * hh;
                     if (tt == 0) {
-                        const uint32_t pb = pfull_b + 8 * es;
+                        const uint32_t pb = efull_b + 8 * es;
                         if (pe_tile) {
                             mbar_arrive_tx(pb, kTile);
                             tma_load_2d(tb + pl.t_bytes, &p.mapPE, col0, (int)(r0 % p.seq_len), pb);
@@ -368,7 +368,7 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
         // positional tiles still in flight after an abort
         if (!ok && tt == 0)
             for (uint32_t i = e > (uint32_t)SE ? e - SE : 0; i < e; ++i)
-                drain_wait(pfull_b + 8 * (i % SE), (i / SE) & 1);
+                drain_wait(efull_b + 8 * (i % SE), (i / SE) & 1);
     }
 
     tc_fence_before();
