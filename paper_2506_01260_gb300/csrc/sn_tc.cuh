@@ -111,17 +111,6 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
     return ok != 0;
 }
 
-// Bounded wait executed by all 32 lanes together: every lane tests the barrier
-// itself (so each observes the completed phase with acquire semantics) and the
-// lanes agree on the outcome.  All 32 lanes must call it.
-__device__ __forceinline__ bool warp_wait_all(uint32_t bar, uint32_t parity, volatile int *abort,
-                                              unsigned int *err)
-{
-    if (__all_sync(0xffffffffu, mbar_test(bar, parity)))
-        return true;
-    return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort, err));
-}
-
 // Short bounded wait used only while draining after an abort.
 __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity)
 {

@@ -211,7 +211,7 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
                 const int blk = block_at(blk0, blk1, j);
                 const uint32_t b = g % kReconAcc;
                 const uint32_t e = 2 * g + grp, es = e % SE, ph = (e / SE) & 1;
-                if (!warp_wait_all(accf_b + 8 * b, (g / kReconAcc) & 1, abort_flag, p.err)) {
+                if (!warp_wait(accf_b + 8 * b, (g / kReconAcc) & 1, abort_flag, p.err)) {
                     ok = false;
                     break;
                 }
@@ -226,7 +226,7 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
                 __syncwarp();
                 if (lane == 0)
                     mbar_arrive(acce_b + 8 * b);
-                if (!warp_wait_all(efull_b + 8 * es, ph, abort_flag, p.err)) {
+                if (!warp_wait(efull_b + 8 * es, ph, abort_flag, p.err)) {
                     ok = false;
                     break;
                 }
