@@ -279,7 +279,9 @@ def config_dict(workload=WORKLOAD):
     return {"workload": desc, "T": wl.T, "d": wl.d, "k": wl.k, "vocab": wl.vocab,
             "seq_len": wl.seq_len, "w_o": list(wo),
             "l2": "flushed before every timed step (512 MiB write)",
-            "parallelism": "independent replicas (one process per GPU)"}
+            "parallelism": "independent replicas (one process per GPU)",
+            "wire": "pinned-host D2H + H2D of C on a copy stream, overlapped with the next "
+                    "compute call; the receiving call waits on it"}
 
 
 # ---- our arm -------------------------------------------------------------------------
@@ -319,27 +321,51 @@ def run_ours(args, world, rank, local, pg):
     names = ["sn_compress_fwd", "sn_decompress_fwd", "sn_compress_bwd", "sn_decompress_bwd",
              "sn_project_weight"]
 
-    def step(ev=None):
-        # ev: list of 2 * len(names) + 1 events bracketing each kernel call
+    # The forward and backward boundary transfers are independent of each
+    # other, so each crosses the wire on its own copy stream while the compute
+    # stream runs the next call (as a pipeline overlaps the activation send of
+    # one microbatch with the gradient work of another); the receiving call
+    # waits on the copy's event.
+    wire_stream = torch.cuda.Stream()
+    sync_ev = [torch.cuda.Event() for _ in range(4)]
+
+    def step(ev=None, wev=None):
+        # ev: 8 events on the compute stream, wev: 4 on the wire stream
         def mark(i):
             if ev is not None:
                 ev[i].record(stream)
+
+        def wmark(i):
+            if wev is not None:
+                wev[i].record(wire_stream)
         mark(0)
         sn.sn_compress_fwd(basis, X, ids, tok, n, pos_emb=pe, out=C)
+        sync_ev[0].record(stream)
         mark(1)
-        sn.sn_wire_send(C, wire_f)
-        sn.sn_wire_recv(wire_f, C_rx)
-        mark(2)
-        sn.sn_decompress_fwd(basis, C_rx, ids, tok, n, pos_emb=pe, out=Xr)
-        mark(3)
+        wire_stream.wait_event(sync_ev[0])
+        wmark(0)
+        sn.sn_wire_send(C, wire_f, stream=wire_stream)
+        sn.sn_wire_recv(wire_f, C_rx, stream=wire_stream)
+        wmark(1)
+        sync_ev[1].record(wire_stream)
         sn.sn_compress_bwd(basis, G, out=Cg)
-        mark(4)
-        sn.sn_wire_send(Cg, wire_b)
-        sn.sn_wire_recv(wire_b, Cg_rx)
-        mark(5)
-        sn.sn_decompress_bwd(basis, Cg_rx, out=Gr)
-        mark(6)
+        sync_ev[2].record(stream)
+        mark(2)
+        wire_stream.wait_event(sync_ev[2])
+        wmark(2)
+        sn.sn_wire_send(Cg, wire_b, stream=wire_stream)
+        sn.sn_wire_recv(wire_b, Cg_rx, stream=wire_stream)
+        wmark(3)
+        sync_ev[3].record(wire_stream)
         sn.sn_project_weight(basis, Wo, out=Wp, workspace=ws)
+        mark(3)
+        stream.wait_event(sync_ev[1])
+        mark(4)
+        sn.sn_decompress_fwd(basis, C_rx, ids, tok, n, pos_emb=pe, out=Xr)
+        mark(5)
+        stream.wait_event(sync_ev[3])
+        mark(6)
+        sn.sn_decompress_bwd(basis, Cg_rx, out=Gr)
         mark(7)
 
     for _ in range(args.warmup):
@@ -349,6 +375,7 @@ def run_ours(args, world, rank, local, pg):
     torch.cuda.synchronize()
 
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(8)] for _ in range(args.steps)]
+    wevs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
     clocks = ClockSampler(local)
     clocks.start()
     barrier(pg)
@@ -357,7 +384,7 @@ def run_ours(args, world, rank, local, pg):
     wall0 = time.perf_counter()
     for i in range(args.steps):
         flush.zero_()
-        step(evs[i])
+        step(evs[i], wevs[i])
     torch.cuda.synchronize()
     wall = time.perf_counter() - wall0
     launches = sn.sn_launch_count() - launches0
@@ -368,12 +395,14 @@ def run_ours(args, world, rank, local, pg):
     per_step = [e[0].elapsed_time(e[7]) for e in evs]          # ms
     seg = {  # ms per launch, averaged over the timed steps
         "sn_compress_fwd": statistics.mean(e[0].elapsed_time(e[1]) for e in evs),
-        "wire_fwd": statistics.mean(e[1].elapsed_time(e[2]) for e in evs),
-        "sn_decompress_fwd": statistics.mean(e[2].elapsed_time(e[3]) for e in evs),
-        "sn_compress_bwd": statistics.mean(e[3].elapsed_time(e[4]) for e in evs),
-        "wire_bwd": statistics.mean(e[4].elapsed_time(e[5]) for e in evs),
-        "sn_decompress_bwd": statistics.mean(e[5].elapsed_time(e[6]) for e in evs),
-        "sn_project_weight": statistics.mean(e[6].elapsed_time(e[7]) for e in evs),
+        "sn_compress_bwd": statistics.mean(e[1].elapsed_time(e[2]) for e in evs),
+        "sn_project_weight": statistics.mean(e[2].elapsed_time(e[3]) for e in evs),
+        "wire_wait": statistics.mean(e[3].elapsed_time(e[4]) + e[5].elapsed_time(e[6])
+                                     for e in evs),
+        "sn_decompress_fwd": statistics.mean(e[4].elapsed_time(e[5]) for e in evs),
+        "sn_decompress_bwd": statistics.mean(e[6].elapsed_time(e[7]) for e in evs),
+        "wire_fwd": statistics.mean(w[0].elapsed_time(w[1]) for w in wevs),
+        "wire_bwd": statistics.mean(w[2].elapsed_time(w[3]) for w in wevs),
     }
     ms = statistics.mean(per_step)
     ms = max_over_ranks(pg, ms, dev)
@@ -448,7 +477,8 @@ def run_ours(args, world, rank, local, pg):
                          "frac": kernels[dom]["gbs"] / hbm, "traffic": traffic,
                          "algorithmic_bytes_per_launch": ab[dom]},
             "kernels": kernels,
-            "wire_ms": {"fwd": seg["wire_fwd"], "bwd": seg["wire_bwd"]},
+            "wire_ms": {"fwd": seg["wire_fwd"], "bwd": seg["wire_bwd"],
+                        "compute_stream_wait": seg["wire_wait"]},
             "boundary_hbm_gbs": sum(ab[nm] for nm in names) / (
                 sum(seg[nm] for nm in names) / 1e3) / 1e9,
             "e2e": e2e_line,

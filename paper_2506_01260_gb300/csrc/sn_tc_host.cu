@@ -120,31 +120,50 @@ void split_blocks(int ntiles, int nblk, int sms, int *bpi, int *chunks)
     *chunks = (nblk + *bpi - 1) / *bpi;
 }
 
-// d-range splits of the projection's first pass.
+// d-range splits of the projection's first pass: the chunk count per item that
+// minimises (rounds of the persistent grid) x (chunks per item), i.e. the
+// longest CTA's chunk count, with at least 8 chunks per item and, among equal
+// costs, the fewest splits (the second pass reads every split's partials).
 void project_splits(int d, int64_t m, int sms, int *splits, int *kc_per)
 {
     const int nkc = (d + BK - 1) / BK;
     const int64_t ntiles = (m + BM - 1) / BM;
-    int want = (int)std::max<int64_t>(1, (2 * sms + ntiles - 1) / ntiles);
-    want = std::min(want, nkc);
-    *kc_per = (nkc + want - 1) / want;
-    *splits = (nkc + *kc_per - 1) / *kc_per;
+    int64_t best = -1;
+    for (int kp = nkc; kp >= 1; --kp) {
+        if (kp < 8 && kp < nkc)
+            break;
+        const int sp = (nkc + kp - 1) / kp;
+        if ((nkc + sp - 1) / sp != kp)
+            continue;                         // same split count as a larger kp
+        const int64_t rounds = (ntiles * sp + sms - 1) / sms;
+        const int64_t cost = rounds * kp;
+        if (best < 0 || cost < best) {
+            best = cost;
+            *kc_per = kp;
+            *splits = sp;
+        }
+    }
 }
 
 size_t align256(size_t v) { return (v + 255) & ~(size_t)255; }
 
+// A^T[c, j] = sum over splits of P[split, c, j], rounded once to bf16 and
+// zero-padded to k64 columns.  One thread per output element; k64 is 64 or 128.
 __global__ void k_sum_partials(const float *__restrict__ P, int splits, int64_t m, int n_pad,
-                               int k, int k64, __nv_bfloat16 *__restrict__ At)
+                               int k, int k64_log2, __nv_bfloat16 *__restrict__ At)
 {
-    const int64_t n = m * k64;
+    const int64_t n = m << k64_log2;
+    const int64_t split_stride = m * n_pad;
     for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n;
          e += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t c = e / k64;
-        const int j = (int)(e % k64);
+        const int64_t c = e >> k64_log2;
+        const int j = (int)(e & ((1 << k64_log2) - 1));
         float s = 0.f;
-        if (j < k)
-            for (int sp = 0; sp < splits; ++sp)
-                s += P[((int64_t)sp * m + c) * n_pad + j];
+        if (j < k) {
+            const float *src = P + c * n_pad + j;
+            for (int sp = 0; sp < splits; ++sp, src += split_stride)
+                s += __ldg(src);
+        }
         At[e] = __float2bfloat16_rn(s);
     }
 }
@@ -293,7 +312,7 @@ cudaError_t tc_project(const sn_basis &b, const __nv_bfloat16 *W, int64_t cols, 
     if (e != cudaSuccess)
         return e;
     // pass 2: sum the partials, round A^T to bf16 [cols, k64] (zero-padded)
-    k_sum_partials<<<2 * sms, 256, 0, s>>>(P, splits, cols, b.n_pad, b.k, b.k64, At);
+    k_sum_partials<<<4 * sms, 256, 0, s>>>(P, splits, cols, b.n_pad, b.k, b.k64 == 64 ? 6 : 7, At);
     count_launch();
     if ((e = cudaGetLastError()) != cudaSuccess)
         return e;
