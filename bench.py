@@ -432,13 +432,46 @@ def run_ours(args, world, rank, local, pg):
         h2d = Xh.numel() * 2 + Gh.numel() * 2 + idsh.numel() * 4
         d2h = Xoh.numel() * 2 + Goh.numel() * 2
 
+        # Host copies ride their own streams so that G's upload overlaps the
+        # forward compress and X' downloads while the gradient recover runs;
+        # every call still waits for the bytes it consumes.
+        h2d_stream = torch.cuda.Stream()
+        d2h_stream = torch.cuda.Stream()
+        cev = [torch.cuda.Event() for _ in range(4)]
+
         def e2e_step():
-            sn.sn_wire_recv(Xh, X)
-            sn.sn_wire_recv(idsh, ids)
-            sn.sn_wire_recv(Gh, G)
-            step()
-            sn.sn_wire_send(Xr, Xoh)
-            sn.sn_wire_send(Gr, Goh)
+            h2d_stream.wait_stream(stream)          # the previous step is done with X, G
+            sn.sn_wire_recv(Xh, X, stream=h2d_stream)
+            sn.sn_wire_recv(idsh, ids, stream=h2d_stream)
+            cev[0].record(h2d_stream)
+            sn.sn_wire_recv(Gh, G, stream=h2d_stream)
+            cev[1].record(h2d_stream)
+            stream.wait_event(cev[0])
+            sn.sn_compress_fwd(basis, X, ids, tok, n, pos_emb=pe, out=C)
+            sync_ev[0].record(stream)
+            wire_stream.wait_event(sync_ev[0])
+            sn.sn_wire_send(C, wire_f, stream=wire_stream)
+            sn.sn_wire_recv(wire_f, C_rx, stream=wire_stream)
+            sync_ev[1].record(wire_stream)
+            stream.wait_event(cev[1])
+            sn.sn_compress_bwd(basis, G, out=Cg)
+            sync_ev[2].record(stream)
+            wire_stream.wait_event(sync_ev[2])
+            sn.sn_wire_send(Cg, wire_b, stream=wire_stream)
+            sn.sn_wire_recv(wire_b, Cg_rx, stream=wire_stream)
+            sync_ev[3].record(wire_stream)
+            sn.sn_project_weight(basis, Wo, out=Wp, workspace=ws)
+            stream.wait_event(sync_ev[1])
+            sn.sn_decompress_fwd(basis, C_rx, ids, tok, n, pos_emb=pe, out=Xr)
+            cev[2].record(stream)
+            d2h_stream.wait_event(cev[2])
+            sn.sn_wire_send(Xr, Xoh, stream=d2h_stream)
+            stream.wait_event(sync_ev[3])
+            sn.sn_decompress_bwd(basis, Cg_rx, out=Gr)
+            cev[3].record(stream)
+            d2h_stream.wait_event(cev[3])
+            sn.sn_wire_send(Gr, Goh, stream=d2h_stream)
+            stream.wait_stream(d2h_stream)          # the step ends when G' is on the host
 
         for _ in range(min(args.warmup, 3)):
             flush.zero_()

@@ -235,14 +235,16 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&v)[16
 }
 __device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
-// Instruction descriptor, kind::f16: bf16 A and B (both K-major), fp32 D,
-// shape M x N; `negate_a` computes D (+)= (-A) B.
-__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool negate_a = false)
+// Instruction descriptor, kind::f16: bf16 A and B (K-major unless
+// `a_mn_major`), fp32 D, shape M x N; `negate_a` computes D (+)= (-A) B.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool negate_a = false,
+                                                  bool a_mn_major = false)
 {
     return (1u << 4)                     // D format: fp32
            | (1u << 7)                   // A format: bf16
            | (1u << 10)                  // B format: bf16
            | ((negate_a ? 1u : 0u) << 13)
+           | ((a_mn_major ? 1u : 0u) << 15)   // A stored MN-major
            | ((uint32_t)(N >> 3) << 17)  // N / 8
            | ((uint32_t)(M >> 4) << 24); // M / 16
 }
@@ -259,6 +261,23 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr)
     d |= (uint64_t)(1024 >> 4) << 32;           // stride byte offset: 8 rows x 128 B
     d |= (uint64_t)1 << 46;                     // descriptor version (sm_100 family)
     d |= (uint64_t)2 << 61;                     // swizzle: 128 B
+    return d;
+}
+
+// Shared-memory matrix descriptor of an MN-major operand in the 128-byte
+// swizzle layout: each K row holds 64 consecutive M (or N) elements in 128
+// bytes, 8-row K groups are `k_group_bytes` apart (stride byte offset) and the
+// next 64 M elements start `mn_block_bytes` later (leading byte offset).
+// Stepping K by 16 rows advances the start address by 2 K groups.
+__device__ __forceinline__ uint64_t sdesc_mn_sw128(uint32_t saddr, uint32_t mn_block_bytes,
+                                                   uint32_t k_group_bytes)
+{
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+    d |= (uint64_t)((mn_block_bytes >> 4) & 0x3FFFu) << 16;
+    d |= (uint64_t)((k_group_bytes >> 4) & 0x3FFFu) << 32;
+    d |= (uint64_t)1 << 46;
+    d |= (uint64_t)2 << 61;
     return d;
 }
 

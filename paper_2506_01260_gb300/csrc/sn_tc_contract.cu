@@ -6,15 +6,15 @@
 //
 // Persistent CTAs walk 128-row tiles in 64-column chunks of d through a ring
 // of shared-memory stages (all operand tiles 128-byte swizzled, K-major):
-//   warp 0     TMA producer: the X/G tile (or raw W tile), the U^T chunk and,
+//   warp 0     TMA producer: the X/G tile (or the W tile, which the MMA reads
+//              MN-major, as two 64-column swizzled boxes), the U^T chunk and,
 //              when a tile's positions are contiguous, the positional tile;
 //   warp 1     allocates TMEM and issues tcgen05.mma (M = 128, N = k padded
 //              to 16, K = 16) into a double-buffered fp32 accumulator.  CMODE_X
 //              accumulates X U - T_fixed[ids] U - P[pos] U: three MMAs per
 //              K-step, the embedding terms with the descriptor's negate-A bit,
 //              so the residual is never rounded;
-//   warps 2-5  CMODE_W: transpose the raw W tile into the K-major A operand;
-//              then drain the accumulator (tcgen05.ld), round once to bf16 and
+//   warps 2-5  drain the accumulator (tcgen05.ld), round once to bf16 and
 //              store each warp's 32 rows of C as one contiguous slab (CMODE_W:
 //              fp32 partial rows);
 //   warps 6-9  CMODE_X: gather the T_fixed rows (and non-contiguous positional
@@ -54,9 +54,9 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
     const int S = p.stages;
     const ContractPlan pl = contract_plan(MODE, p.n_pad, p.k, p.has_pe, S);
     const uint32_t bar = base + pl.bar_off;
-    const uint32_t full_b = bar, rr_b = bar + 8 * S, empty_b = bar + 16 * S;
-    const uint32_t accf_b = bar + 24 * S, acce_b = accf_b + 16, drain_b = acce_b + 16;
-    uint32_t *tmem_slot = (uint32_t *)(smem + pl.bar_off + 8 * (3 * S + 5));
+    const uint32_t full_b = bar, empty_b = bar + 8 * S;
+    const uint32_t accf_b = bar + 16 * S, acce_b = accf_b + 16, drain_b = acce_b + 16;
+    uint32_t *tmem_slot = (uint32_t *)(smem + pl.bar_off + 8 * (2 * S + 5));
     volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t tmem_cols = 2 * p.acc_stride;
@@ -64,7 +64,6 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
             mbar_init(full_b + 8 * s, MODE == CMODE_X ? 1 + 128 : 1);   // TMA + gather threads
-            mbar_init(rr_b + 8 * s, 4);
             mbar_init(empty_b + 8 * s, 1);
         }
         for (int b = 0; b < 2; ++b) {
@@ -103,8 +102,7 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
                                                : tile_row0(tile, p.reorder, p.batches, p.seq_len);
             const bool pe_tile = MODE == CMODE_X && p.has_pe && !p.has_pos &&
                                  (r0 % p.seq_len) + BM <= p.seq_len;
-            const uint32_t tx = MODE == CMODE_W ? pl.raw_bytes + pl.u_bytes
-                                                : pl.a_bytes + pl.u_bytes + (pe_tile ? kTile : 0);
+            const uint32_t tx = pl.a_bytes + pl.u_bytes + (pe_tile ? kTile : 0);
             for (int j = 0; j < kc1 - kc0; ++j, ++g) {
                 const int kc = chunk_at(kc0, kc1, j);
                 const int s = g % S;
@@ -117,10 +115,12 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
                 const uint32_t fb = full_b + 8 * s;
                 if (lane == 0) {
                     mbar_arrive_tx(fb, tx);
-                    if (MODE == CMODE_W)
-                        tma_load_2d(st + pl.a_bytes + pl.u_bytes, &p.mapA, (int)r0, kc * BK, fb);
-                    else
+                    if (MODE == CMODE_W) {   // W[kc*64 .. +64, r0 .. r0+128): d rows x c
+                        tma_load_2d(st, &p.mapA, (int)r0, kc * BK, fb);
+                        tma_load_2d(st + kTile / 2, &p.mapA, (int)r0 + 64, kc * BK, fb);
+                    } else {
                         tma_load_2d(st, &p.mapA, kc * BK, (int)r0, fb);
+                    }
                     tma_load_2d(st + pl.a_bytes, &p.mapU, kc * BK, 0, fb);
                     if (pe_tile)
                         tma_load_2d(st + pl.a_bytes + pl.u_bytes + pl.raw_bytes, &p.mapPE,
@@ -137,7 +137,7 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
-            const uint32_t idesc = idesc_bf16(BM, p.n_pad);
+            const uint32_t idesc = idesc_bf16(BM, p.n_pad, false, MODE == CMODE_W);
             const uint32_t idesc_neg = idesc_bf16(BM, p.n_pad, true);
             uint32_t g = 0, it = 0;
             bool ok = true;
@@ -155,8 +155,7 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
                 for (int j = 0; j < kc1 - kc0; ++j, ++g) {
                     const int s = g % S;
                     const uint32_t n = g / S;
-                    const uint32_t wb = (MODE == CMODE_W ? rr_b : full_b) + 8 * s;
-                    if (!mbar_wait(wb, n & 1, abort_flag, p.err)) {
+                    if (!mbar_wait(full_b + 8 * s, n & 1, abort_flag, p.err)) {
                         ok = false;
                         break;
                     }
@@ -168,7 +167,12 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
 #pragma unroll
                     for (int kk = 0; kk < BK / 16; ++kk) {
                         const uint64_t bd = sdesc_sw128(ub + kk * 32);
-                        mma_bf16(d_tmem, sdesc_sw128(st + kk * 32), bd, idesc,
+                        // A: K-major rows (X, G), or the W tile MN-major (16 d rows
+                        // per step; the second 64 columns 8 KB on)
+                        const uint64_t ad = MODE == CMODE_W
+                                                ? sdesc_mn_sw128(st + kk * 2048, kTile / 2, 1024)
+                                                : sdesc_sw128(st + kk * 32);
+                        mma_bf16(d_tmem, ad, bd, idesc,
                                  (j > 0 || kk > 0) ? 1u : 0u);
                         if (MODE == CMODE_X) {   // - T_fixed[ids] U - P[pos] U
                             const uint32_t tb = ub + pl.u_bytes;
@@ -192,51 +196,13 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
     } else if (warp < 6) {
         // ------------------------------------------------------------ epilogue warps
         const int q = warp & 3;              // TMEM lane quarter of this warp
-        const int tt = threadIdx.x - 64;     // 0..127
         const int row = 32 * q + lane;
-        uint32_t g = 0, it = 0;
+        uint32_t it = 0;
         bool ok = true;
         for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++it) {
             const int tile = item / p.splits, split = item % p.splits;
-            const int kc0 = split * p.kc_per_item;
-            const int kc1 = min(kc0 + p.kc_per_item, kc_total);
             const int64_t r0 = MODE == CMODE_W ? (int64_t)tile * BM
                                                : tile_row0(tile, p.reorder, p.batches, p.seq_len);
-            if (MODE == CMODE_W) {
-                for (int j = 0; j < kc1 - kc0; ++j, ++g) {
-                    const int s = g % S;
-                    const uint32_t n = g / S;
-                    if (!warp_wait(full_b + 8 * s, n & 1, abort_flag, p.err)) {
-                        ok = false;
-                        break;
-                    }
-                    // raw W tile [64 d][128 c] -> A operand [128 c][64 d]
-                    const uint32_t st = base + s * pl.stage_bytes;
-                    const uint32_t raw = st + pl.a_bytes + pl.u_bytes;
-#pragma unroll
-                    for (int c = 0; c < 8; ++c) {
-                        uint32_t w[4];
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            unsigned short lo, hi;
-                            asm volatile("ld.shared.u16 %0, [%1];"
-                                         : "=h"(lo)
-                                         : "r"(raw + (8 * c + 2 * e) * 256 + tt * 2));
-                            asm volatile("ld.shared.u16 %0, [%1];"
-                                         : "=h"(hi)
-                                         : "r"(raw + (8 * c + 2 * e + 1) * 256 + tt * 2));
-                            w[e] = (uint32_t)lo | ((uint32_t)hi << 16);
-                        }
-                        sts128(st + sw128(tt, c), make_uint4(w[0], w[1], w[2], w[3]));
-                    }
-                    fence_async_smem();
-                    __syncwarp();
-                    if (lane == 0)
-                        mbar_arrive(rr_b + 8 * s);
-                }
-                if (!ok)
-                    break;
-            }
             // ---- accumulator -> output
             const uint32_t b = it & 1, nb = it >> 1;
             if (!warp_wait(accf_b + 8 * b, nb & 1, abort_flag, p.err)) {

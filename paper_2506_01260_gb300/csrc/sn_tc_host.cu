@@ -289,7 +289,7 @@ cudaError_t tc_project(const sn_basis &b, const __nv_bfloat16 *W, int64_t cols, 
     // pass 1: fp32 partials of A^T = (U^T W)^T over d-ranges
     ContractParams p;
     std::memset(&p, 0, sizeof p);
-    bool ok = map2d(&p.mapA, W, cols, b.d, (uint64_t)ld * 2, BM, BK, false) &&
+    bool ok = map2d(&p.mapA, W, cols, b.d, (uint64_t)ld * 2, 64, BK, true) &&
               map2d(&p.mapU, b.ut16, b.d, b.n_pad, (uint64_t)b.d * 2, BK, b.n_pad, true);
     p.mapPE = p.mapA;
     if (!ok)

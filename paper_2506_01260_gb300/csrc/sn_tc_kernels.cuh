@@ -20,7 +20,7 @@ constexpr uint32_t kTile = BM * 128;      // one [128 x 64] bf16 swizzled tile
 enum { CMODE_G = 0, CMODE_X = 1, CMODE_W = 2 };
 
 struct ContractParams {
-    CUtensorMap mapA;    // X or G [T, d] (SW128, box 64 x 128) | W [d, m] (plain, box 128 x 64)
+    CUtensorMap mapA;    // X or G [T, d] (SW128, box 64 x 128) | W [d, m] (SW128, box 64 x 64)
     CUtensorMap mapU;    // U^T padded [n_pad, d] (SW128, box 64 x n_pad)
     CUtensorMap mapPE;   // P [seq_len, d] (SW128, box 64 x 128), contiguous positions
     const __nv_bfloat16 *tok;   // T_fixed [vocab, d], rows gathered with cp.async
@@ -55,14 +55,13 @@ __host__ __device__ inline ContractPlan contract_plan(int mode, int n_pad, int k
     ContractPlan p;
     p.a_bytes = kTile;
     p.u_bytes = (uint32_t)n_pad * 128;
-    p.raw_bytes = (mode == CMODE_X || mode == CMODE_W) ? kTile : 0;   // T_fixed rows | raw W
+    p.raw_bytes = (mode == CMODE_X) ? kTile : 0;   // T_fixed rows
     p.pe_bytes = (mode == CMODE_X && has_pe) ? kTile : 0;
     p.stage_bytes = p.a_bytes + p.u_bytes + p.raw_bytes + p.pe_bytes;
     p.cst_bytes = (mode == CMODE_W) ? 0 : (((uint32_t)BM * k * 2 + 1023) & ~1023u);
     p.bar_off = (uint32_t)stages * p.stage_bytes + p.cst_bytes;
-    p.total = p.bar_off + 8 * (3 * stages + 5) + 16 + 1024;   // + alignment slack
-    p.tx_bytes = (mode == CMODE_W) ? p.raw_bytes + p.u_bytes
-                                   : p.a_bytes + p.u_bytes + p.raw_bytes + p.pe_bytes;
+    p.total = p.bar_off + 8 * (2 * stages + 5) + 16 + 1024;   // + alignment slack
+    p.tx_bytes = p.a_bytes + p.u_bytes + p.pe_bytes;
     return p;
 }
 
