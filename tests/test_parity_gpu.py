@@ -303,3 +303,35 @@ def test_argument_errors(sn):
     with pytest.raises(sn.SNError):           # k > d
         sn.Basis(torch.zeros(16, 17, device="cuda"))
     basis.destroy()
+
+
+@pytest.mark.parametrize("layout", ["ragged", "position_major"])
+def test_more_tiles_than_sms(sn, oracle, layout):
+    """More row tiles than SMs, so every persistent CTA takes several tiles and
+    a few take one more (ragged last tile, and the position-block-major tile
+    order); every row of C must come out."""
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    if layout == "ragged":
+        T, n = (sms + 9) * 128 - 50, 128          # 9 tiles past one per SM, the last ragged
+    else:
+        T, n = (sms + 8) * 128, 256               # 2-tile sequences, tiles run position-major
+    d, k, vocab = 128, 24, 600
+    inp = case_inputs("tail_" + layout, T, n, d, k, vocab, "bf16", seed=11)
+    basis = sn.Basis(dev(inp["U"]))
+    X, tok, pe, ids, G = (dev(inp["X"]), dev(inp["tok_emb"]), dev(inp["pos_emb"]),
+                          dev(inp["ids"]), dev(inp["G"]))
+    fullC, C = guarded((T, k), X.dtype)
+    sn.sn_compress_fwd(basis, X, ids, tok, n, pos_emb=pe, out=C)
+    fullCg, Cg = guarded((T, k), X.dtype)
+    sn.sn_compress_bwd(basis, G, out=Cg)
+    sn.sn_check_errors(basis)
+    assert guards_intact(fullC) and guards_intact(fullCg)
+    _, C64, st = oracle.compress_fwd(inp["X"], inp["ids"], inp["tok_emb"], inp["U"], n,
+                                     pos_emb=inp["pos_emb"])
+    assert st == 0
+    assert rel_fro(host(C), C64) <= TOL["bf16"]
+    _, Cg64, _ = oracle.compress_bwd(inp["G"], inp["U"])
+    assert rel_fro(host(Cg), Cg64) <= TOL["bf16"]
+    # every row is covered: no row of C left at the guard fill or zero
+    assert np.all(np.abs(widen(host(C))).sum(axis=1) > 0)
+    basis.destroy()
