@@ -50,6 +50,7 @@ def parse():
                     help="target CPU time of the oracle baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-next", action="store_true", help="skip the NEXT-row measurements")
     ap.add_argument("--workload", choices=sorted(PROFILE_WORKLOADS), default=WORKLOAD,
                     help="large (default, the benchmark) or a smaller case for profiling")
     return ap.parse_args()
@@ -418,6 +419,40 @@ def run_ours(args, world, rank, local, pg):
     dom = max(names, key=lambda nm: seg[nm])
     traffic = measured_traffic(dom) if args.workload == WORKLOAD else None
 
+    # ---- NEXT f3, reported apart from the step: compress with projected tables
+    nxt = None
+    if not args.no_next:
+        ev0 = torch.cuda.Event(enable_timing=True)
+        ev1 = torch.cuda.Event(enable_timing=True)
+        ev0.record(stream)
+        TU, PU = sn.sn_project_tables(basis, tok, pos_emb=pe)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        build_ms = ev0.elapsed_time(ev1)
+        Cp = torch.empty_like(C)
+        for _ in range(args.warmup):
+            flush.zero_()
+            sn.sn_compress_fwd_projected(basis, X, ids, TU, n, PU=PU, out=Cp)
+        pev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(min(args.steps, 50))]
+        for a_, b_ in pev:
+            flush.zero_()
+            a_.record(stream)
+            sn.sn_compress_fwd_projected(basis, X, ids, TU, n, PU=PU, out=Cp)
+            b_.record(stream)
+        torch.cuda.synchronize()
+        sn.sn_check_errors(basis)
+        pms = max_over_ranks(pg, statistics.mean(a_.elapsed_time(b_) for a_, b_ in pev), dev)
+        pab = 2 * T * d + 4 * u * k + 4 * min(n, T) * k + 4 * d * k + 2 * T * k
+        nxt = {"f3_projected_compress": {
+            "ms": pms, "algorithmic_bytes": pab, "gbs": pab / (pms / 1e3) / 1e9,
+            "frac": pab / (pms / 1e3) / 1e9 / hbm,
+            "table_build_ms": build_ms,
+            "speedup_vs_sn_compress_fwd": seg["sn_compress_fwd"] / pms,
+            "note": "C = X U - (T_fixed U)[ids] - (P U)[pos] with the tables projected once "
+                    "(sn_project_tables); same C as sn_compress_fwd"}}
+        del TU, PU, Cp
+
     # ---- end to end through the C ABI with host buffers ----
     e2e_line = None
     if not args.no_e2e:
@@ -524,6 +559,7 @@ def run_ours(args, world, rank, local, pg):
                         "compute_stream_wait": seg["wire_wait"]},
             "boundary_hbm_gbs": sum(ab[nm] for nm in names) / (
                 sum(seg[nm] for nm in names) / 1e3) / 1e9,
+            "next": nxt,
             "e2e": e2e_line,
             "gpu_launches": launches,
             "unique_ids": u,

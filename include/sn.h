@@ -137,6 +137,40 @@ sn_status sn_project_weight_noalloc(sn_basis_t basis, sn_dtype dtype, const void
                                     int64_t rows, int64_t cols, int64_t ld, void *W_out,
                                     sn_stream_t stream);
 
+/* ---- Projected embedding tables (a variant of the forward compress) ----------
+ * Because the compress of Sec. 4.3.1, Eq. (subtract), is linear,
+ *   (X - T_fixed[ids] - P[p]) U = X U - (T_fixed U)[ids] - (P U)[p],
+ * and T_fixed is fixed for the whole run (Sec. 4.3.1: sent to every node once),
+ * the embedding rows can be projected once per U and the per-step compress then
+ * reads k-wide rows instead of d-wide ones.  bf16 only (SN_ERR_UNSUPPORTED for
+ * SN_F32). */
+
+/* TU = T_fixed U (fp32 [vocab, k], row-major) and, when pos_emb is non-NULL,
+ * PU = P U (fp32 [seq_len, k]).  tok_emb [vocab, d], pos_emb [seq_len, d];
+ * pos_emb and PU are both NULL or both non-NULL.  Accumulated in fp32 from the
+ * bf16 tables and the bf16 copy of U, never rounded. */
+sn_status sn_project_tables(sn_basis_t basis, sn_dtype dtype, const void *tok_emb, int64_t vocab,
+                            const void *pos_emb, int32_t seq_len, float *TU, float *PU,
+                            sn_stream_t stream);
+
+/* C[t, :] = X[t, :] U - TU[ids[t], :] - PU[p(t), :], one rounding to bf16 (the
+ * same C as sn_compress_fwd with the tables TU, PU were projected from).
+ * Arguments as in sn_compress_fwd with TU [vocab, k] and PU [seq_len, k] (or
+ * NULL: nothing positional is subtracted and `pos` is ignored) in place of the
+ * d-wide tables.  Invalid ids and positions behave as in sn_compress_fwd. */
+sn_status sn_compress_fwd_projected(sn_basis_t basis, sn_dtype dtype, const void *X,
+                                    const int32_t *ids, const int32_t *pos, int64_t T,
+                                    int32_t seq_len, const float *TU, int64_t vocab,
+                                    const float *PU, void *C, sn_stream_t stream);
+
+/* The low-rank part of the token embeddings, Sec. 4.3.1: T_S = T_fixed U U^T
+ * (bf16 [vocab, d]; computed as (T_fixed U) U^T with T_fixed U rounded once to
+ * bf16 in between, like the weight projection).  `workspace` is device memory of
+ * at least sn_wire_bytes(basis, dtype, vocab) bytes, used only during the call.
+ * T_S may not overlap tok_emb or the workspace. */
+sn_status sn_build_ts(sn_basis_t basis, sn_dtype dtype, const void *tok_emb, int64_t vocab,
+                      void *T_S, void *workspace, size_t workspace_bytes, sn_stream_t stream);
+
 /* Bytes on the wire for T tokens: T * k * element size (Sec. 4.3: k/d of X). */
 sn_status sn_wire_bytes(sn_basis_t basis, sn_dtype dtype, int64_t T, size_t *bytes);
 

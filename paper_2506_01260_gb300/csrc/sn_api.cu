@@ -280,6 +280,74 @@ sn_status sn_project_weight(sn_basis_t b, sn_dtype dt, const void *W, int64_t ro
                                       (__nv_bfloat16 *)W_out, ws, s));
 }
 
+sn_status sn_project_tables(sn_basis_t b, sn_dtype dt, const void *tok, int64_t vocab,
+                            const void *pe, int32_t seq_len, float *TU, float *PU,
+                            sn_stream_t stream)
+{
+    sn_status st = check_basis(b, dt);
+    if (st != SN_OK)
+        return st;
+    if (dt != SN_BF16)
+        return SN_ERR_UNSUPPORTED;
+    if (vocab <= 0 || vocab >= kMaxRows || !tok || !TU || (pe == nullptr) != (PU == nullptr) ||
+        (pe && (seq_len <= 0 || seq_len >= kMaxRows)))
+        return SN_ERR_INVALID_ARG;
+    if (!aligned(tok, 16) || !aligned(TU, 16) || (pe && (!aligned(pe, 16) || !aligned(PU, 16))))
+        return SN_ERR_ALIGNMENT;
+    if (overlap(tok, (size_t)vocab * b->d * 2, TU, (size_t)vocab * b->k * 4) ||
+        (pe && (overlap(pe, (size_t)seq_len * b->d * 2, PU, (size_t)seq_len * b->k * 4) ||
+                overlap(TU, (size_t)vocab * b->k * 4, PU, (size_t)seq_len * b->k * 4))))
+        return SN_ERR_INVALID_ARG;
+    cudaStream_t s = (cudaStream_t)stream;
+    cudaError_t e = sn::tc_contract_f32(*b, (const __nv_bfloat16 *)tok, vocab, TU, s);
+    if (e == cudaSuccess && pe)
+        e = sn::tc_contract_f32(*b, (const __nv_bfloat16 *)pe, seq_len, PU, s);
+    return cuda_status(e);
+}
+
+sn_status sn_compress_fwd_projected(sn_basis_t b, sn_dtype dt, const void *X, const int32_t *ids,
+                                    const int32_t *pos, int64_t T, int32_t seq_len,
+                                    const float *TU, int64_t vocab, const float *PU, void *C,
+                                    sn_stream_t stream)
+{
+    sn_status st = check_fwd(b, dt, X, ids, pos, T, seq_len, TU, vocab, PU, C, b ? b->d : 0,
+                             b ? b->k : 0);
+    if (st != SN_OK || T == 0)
+        return st;
+    if (dt != SN_BF16)
+        return SN_ERR_UNSUPPORTED;
+    return cuda_status(sn::tc_compress_projected(*b, (const __nv_bfloat16 *)X, ids, pos, T,
+                                                 seq_len, TU, vocab, PU, (__nv_bfloat16 *)C,
+                                                 (cudaStream_t)stream));
+}
+
+sn_status sn_build_ts(sn_basis_t b, sn_dtype dt, const void *tok, int64_t vocab, void *T_S,
+                      void *ws, size_t ws_bytes, sn_stream_t stream)
+{
+    sn_status st = check_basis(b, dt);
+    if (st != SN_OK)
+        return st;
+    if (dt != SN_BF16)
+        return SN_ERR_UNSUPPORTED;
+    if (vocab <= 0 || vocab >= kMaxRows || !tok || !T_S || !ws)
+        return SN_ERR_INVALID_ARG;
+    const size_t table = (size_t)vocab * b->d * 2, coeff = (size_t)vocab * b->k * 2;
+    if (ws_bytes < coeff)
+        return SN_ERR_INVALID_ARG;
+    if (!aligned(tok, 16) || !aligned(T_S, 16) || !aligned(ws, 16))
+        return SN_ERR_ALIGNMENT;
+    if (overlap(tok, table, T_S, table) || overlap(tok, table, ws, coeff) ||
+        overlap(T_S, table, ws, coeff))
+        return SN_ERR_INVALID_ARG;
+    cudaStream_t s = (cudaStream_t)stream;
+    sn::TcArgs a{(const __nv_bfloat16 *)tok, nullptr, nullptr, nullptr, nullptr,
+                 (__nv_bfloat16 *)ws, vocab, 1, 1, false};
+    cudaError_t e = sn::tc_compress(*b, a, s);
+    if (e == cudaSuccess)
+        e = sn::tc_decompress(*b, a, (__nv_bfloat16 *)T_S, s);
+    return cuda_status(e);
+}
+
 sn_status sn_wire_bytes(sn_basis_t b, sn_dtype dt, int64_t T, size_t *bytes)
 {
     if (!b || !bytes || T < 0 || (dt != SN_BF16 && dt != SN_F32))

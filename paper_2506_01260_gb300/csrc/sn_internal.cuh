@@ -69,5 +69,13 @@ cudaError_t tc_decompress(const sn_basis &b, const TcArgs &a, __nv_bfloat16 *X_o
 cudaError_t tc_project(const sn_basis &b, const __nv_bfloat16 *W, int64_t cols, int64_t ld,
                        __nv_bfloat16 *W_out, void *workspace, cudaStream_t s);
 size_t tc_project_workspace(const sn_basis &b, int64_t cols);
+// out[r, :] = A[r, :] U in fp32 (projected tables: T_fixed U, P U)
+cudaError_t tc_contract_f32(const sn_basis &b, const __nv_bfloat16 *A, int64_t rows, float *out,
+                            cudaStream_t s);
+// C = X U - TU[ids] - PU[pos] (PU may be null)
+cudaError_t tc_compress_projected(const sn_basis &b, const __nv_bfloat16 *X, const int32_t *ids,
+                                  const int32_t *pos, int64_t T, int seq_len, const float *TU,
+                                  int64_t vocab, const float *PU, __nv_bfloat16 *C,
+                                  cudaStream_t s);
 
 }  // namespace sn

@@ -3,6 +3,8 @@
 //   CMODE_X  C[t, :] = (X[t, :] - T_fixed[id_t, :] - P[p_t, :]) U     Sec. 4.3.1, Eq. (subtract)
 //   CMODE_G  C[t, :] = G[t, :] U                                       Sec. 4.4, Eq. (grad_compress)
 //   CMODE_W  A^T[c, :] = W[:, c]^T U  (fp32 partials over a d-range)    first pass of W' = U (U^T W)
+//   CMODE_GF C[r, :] = A[r, :] U, fp32 out                            projected tables T_fixed U, P U
+//   CMODE_XP C[t, :] = X[t, :] U - TU[id_t, :] - PU[p_t, :]             Eq. (subtract), projected tables
 //
 // Persistent CTAs walk 128-row tiles in 64-column chunks of d through a ring
 // of shared-memory stages (all operand tiles 128-byte swizzled, K-major):
@@ -232,18 +234,26 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
             } else {
                 const int64_t t = r0 + row;
                 bool bad = false;
-                if (MODE == CMODE_X && t < p.rows) {
+                int64_t tu_off = 0, pu_off = -1;   // XP: this row's TU and PU rows
+                if ((MODE == CMODE_X || MODE == CMODE_XP) && t < p.rows) {
                     const int id = p.ids[t];
                     bad = id < 0 || id >= p.vocab;
-                    if (p.has_pe && p.has_pos) {
-                        const int ps = p.pos[t];
+                    int ps = 0;
+                    if (p.has_pe) {
+                        ps = p.has_pos ? p.pos[t] : (int)(t % p.seq_len);
                         bad = bad || ps < 0 || ps >= p.seq_len;
                     }
                     if (bad)
                         atomicOr(p.err, SN_EBIT_BAD_ID);
+                    else if (MODE == CMODE_XP) {
+                        tu_off = (int64_t)id * p.k;
+                        if (p.has_pe)
+                            pu_off = (int64_t)ps * p.k;
+                    }
                 }
-                __nv_bfloat16 *cst = (__nv_bfloat16 *)(smem + (size_t)S * pl.stage_bytes);
-                __nv_bfloat16 *crow = cst + (size_t)row * p.k;
+                // stage the rows (bf16, or fp32 in GF mode) for contiguous slab stores
+                constexpr int es = MODE == CMODE_GF ? 4 : 2;
+                uint8_t *cst = smem + (size_t)S * pl.stage_bytes;
                 for (int cc = 0; cc < p.n_pad / 16; ++cc) {
                     float v[16];
                     tmem_ld16(taddr + 16 * cc, v);
@@ -251,25 +261,39 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
 #pragma unroll
                     for (int j = 0; j < 16; ++j) {
                         const int col = 16 * cc + j;
-                        if (col < p.k)
-                            crow[col] = __float2bfloat16_rn(bad ? 0.f : v[j]);
+                        if (col < p.k) {
+                            if (MODE == CMODE_GF) {
+                                ((float *)cst)[(size_t)row * p.k + col] = v[j];
+                            } else {
+                                float x = v[j];
+                                if (MODE == CMODE_XP && !bad) {
+                                    x -= __ldg(p.TU + tu_off + col);
+                                    if (pu_off >= 0)
+                                        x -= __ldg(p.PU + pu_off + col);
+                                }
+                                ((__nv_bfloat16 *)cst)[(size_t)row * p.k + col] =
+                                    __float2bfloat16_rn(bad ? 0.f : x);
+                            }
+                        }
                     }
                 }
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0)
                     mbar_arrive(acce_b + 8 * b);
-                // this warp's 32 rows are one contiguous slab of 32 * k bf16 in C
+                // this warp's 32 rows are one contiguous slab of 32 * k elements of the output
                 const int64_t wr0 = r0 + 32 * q;
                 const int64_t nrows = p.rows - wr0 < 32 ? p.rows - wr0 : 32;
                 if (nrows > 0) {
-                    const uint32_t src = smem_u32(cst + (size_t)32 * q * p.k);
-                    uint8_t *dst = (uint8_t *)(p.C + wr0 * p.k);
-                    const int nbytes = (int)nrows * p.k * 2;
+                    const uint32_t src = smem_u32(cst + (size_t)32 * q * p.k * es);
+                    uint8_t *dst = MODE == CMODE_GF ? (uint8_t *)(p.Cf + wr0 * p.k)
+                                                    : (uint8_t *)(p.C + wr0 * p.k);
+                    const int nbytes = (int)nrows * p.k * es;
                     for (int v = lane; v < nbytes / 16; v += 32)
                         *(uint4 *)(dst + 16 * v) = lds128(src + 16 * v);
-                    for (int e = (nbytes / 16) * 8 + lane; e < nbytes / 2; e += 32)
-                        ((__nv_bfloat16 *)dst)[e] = cst[(size_t)32 * q * p.k + e];
+                    for (int e = (nbytes / 16) * 16 + 2 * lane; e < nbytes; e += 64)
+                        *(unsigned short *)(dst + e) =
+                            *(const unsigned short *)(cst + (size_t)32 * q * p.k * es + e);
                 }
                 __syncwarp();
             }
@@ -333,26 +357,30 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
 
 }  // namespace
 
+namespace {
+
+template <int MODE>
+cudaError_t launch_mode(const ContractParams &p, int grid, uint32_t smem, cudaStream_t s)
+{
+    cudaError_t e =
+        cudaFuncSetAttribute(k_contract<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e == cudaSuccess)
+        k_contract<MODE><<<grid, contract_threads(MODE), smem, s>>>(p);
+    return e;
+}
+
+}  // namespace
+
 cudaError_t launch_contract(int mode, const ContractParams &p, int grid, cudaStream_t s)
 {
     const ContractPlan pl = contract_plan(mode, p.n_pad, p.k, p.has_pe, p.stages);
-    const int threads = contract_threads(mode);
     cudaError_t e;
-    if (mode == CMODE_X) {
-        e = cudaFuncSetAttribute(k_contract<CMODE_X>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 pl.total);
-        if (e == cudaSuccess)
-            k_contract<CMODE_X><<<grid, threads, pl.total, s>>>(p);
-    } else if (mode == CMODE_G) {
-        e = cudaFuncSetAttribute(k_contract<CMODE_G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 pl.total);
-        if (e == cudaSuccess)
-            k_contract<CMODE_G><<<grid, threads, pl.total, s>>>(p);
-    } else {
-        e = cudaFuncSetAttribute(k_contract<CMODE_W>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 pl.total);
-        if (e == cudaSuccess)
-            k_contract<CMODE_W><<<grid, threads, pl.total, s>>>(p);
+    switch (mode) {
+    case CMODE_X: e = launch_mode<CMODE_X>(p, grid, pl.total, s); break;
+    case CMODE_G: e = launch_mode<CMODE_G>(p, grid, pl.total, s); break;
+    case CMODE_W: e = launch_mode<CMODE_W>(p, grid, pl.total, s); break;
+    case CMODE_GF: e = launch_mode<CMODE_GF>(p, grid, pl.total, s); break;
+    default: e = launch_mode<CMODE_XP>(p, grid, pl.total, s); break;
     }
     if (e != cudaSuccess)
         return e;

@@ -218,6 +218,70 @@ cudaError_t tc_compress(const sn_basis &b, const TcArgs &a, cudaStream_t s)
     return launch_contract(mode, p, grid, s);
 }
 
+namespace {
+
+// Contraction parameters shared by the projected-table calls: A [rows, d]
+// K-major through TMA, U^T chunks, no embedding tiles.
+bool contract_plain(tc::ContractParams &p, const sn_basis &b, const __nv_bfloat16 *A,
+                    int64_t rows)
+{
+    using namespace tc;
+    std::memset(&p, 0, sizeof p);
+    if (!map2d(&p.mapA, A, b.d, rows, (uint64_t)b.d * 2, BK, BM, true) ||
+        !map2d(&p.mapU, b.ut16, b.d, b.n_pad, (uint64_t)b.d * 2, BK, b.n_pad, true))
+        return false;
+    p.mapPE = p.mapA;
+    p.err = b.err;
+    p.rows = rows;
+    p.vocab = 1;
+    p.seq_len = 1;
+    p.d = b.d;
+    p.k = b.k;
+    p.n_pad = b.n_pad;
+    p.acc_stride = pow2_at_least(b.n_pad, 32);
+    p.nkc = (b.d + BK - 1) / BK;
+    p.kc_per_item = p.nkc;
+    p.splits = 1;
+    p.ntiles = (int)((rows + BM - 1) / BM);
+    return true;
+}
+
+}  // namespace
+
+cudaError_t tc_contract_f32(const sn_basis &b, const __nv_bfloat16 *A, int64_t rows, float *out,
+                            cudaStream_t s)
+{
+    using namespace tc;
+    ContractParams p;
+    if (!contract_plain(p, b, A, rows))
+        return cudaErrorInvalidValue;
+    p.Cf = out;
+    p.stages = contract_stages(CMODE_GF, b.n_pad, b.k, 0);
+    return launch_contract(CMODE_GF, p, std::min(p.ntiles, sm_count(current_device())), s);
+}
+
+cudaError_t tc_compress_projected(const sn_basis &b, const __nv_bfloat16 *X, const int32_t *ids,
+                                  const int32_t *pos, int64_t T, int seq_len, const float *TU,
+                                  int64_t vocab, const float *PU, __nv_bfloat16 *C,
+                                  cudaStream_t s)
+{
+    using namespace tc;
+    ContractParams p;
+    if (!contract_plain(p, b, X, T))
+        return cudaErrorInvalidValue;
+    p.C = C;
+    p.ids = ids;
+    p.pos = PU ? pos : nullptr;
+    p.TU = TU;
+    p.PU = PU;
+    p.vocab = vocab;
+    p.seq_len = seq_len;
+    p.has_pe = PU != nullptr;
+    p.has_pos = PU != nullptr && pos != nullptr;
+    p.stages = contract_stages(CMODE_XP, b.n_pad, b.k, 0);
+    return launch_contract(CMODE_XP, p, std::min(p.ntiles, sm_count(current_device())), s);
+}
+
 cudaError_t tc_decompress(const sn_basis &b, const TcArgs &a, __nv_bfloat16 *X_out,
                           cudaStream_t s)
 {

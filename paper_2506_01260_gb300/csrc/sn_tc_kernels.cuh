@@ -17,7 +17,13 @@ constexpr uint32_t kSmemLimit = 232448;   // 227 KB per CTA
 constexpr uint32_t kTile = BM * 128;      // one [128 x 64] bf16 swizzled tile
 
 // ---- contraction: out[r, :] = A[r, :] . U   (A = X - E, G, or W^T) -----------
-enum { CMODE_G = 0, CMODE_X = 1, CMODE_W = 2 };
+enum {
+    CMODE_G = 0,    // C = G U (bf16 out)
+    CMODE_X = 1,    // C = (X - T_fixed[ids] - P[pos]) U (bf16 out)
+    CMODE_W = 2,    // fp32 partials of W^T U over d-ranges (projection pass 1)
+    CMODE_GF = 3,   // C = A U, fp32 out (projected tables T_fixed U, P U)
+    CMODE_XP = 4    // C = X U - TU[ids] - PU[pos] (bf16 out, projected tables)
+};
 
 struct ContractParams {
     CUtensorMap mapA;    // X or G [T, d] (SW128, box 64 x 128) | W [d, m] (SW128, box 64 x 64)
@@ -27,8 +33,11 @@ struct ContractParams {
     const __nv_bfloat16 *pe;    // P [seq_len, d], gathered when positions are not contiguous
     const int32_t *ids;
     const int32_t *pos;
-    __nv_bfloat16 *C;    // [T, k] output (G, X modes)
+    __nv_bfloat16 *C;    // [T, k] output (G, X, XP modes)
     float *P;            // [splits, rows, n_pad] fp32 partial output (W mode)
+    float *Cf;           // [rows, k] fp32 output (GF mode)
+    const float *TU;     // [vocab, k] fp32 T_fixed U (XP mode)
+    const float *PU;     // [seq_len, k] fp32 P U (XP mode) or null
     unsigned int *err;
     int64_t rows;        // T, or m (columns of W)
     int64_t vocab;
@@ -58,7 +67,9 @@ __host__ __device__ inline ContractPlan contract_plan(int mode, int n_pad, int k
     p.raw_bytes = (mode == CMODE_X) ? kTile : 0;   // T_fixed rows
     p.pe_bytes = (mode == CMODE_X && has_pe) ? kTile : 0;
     p.stage_bytes = p.a_bytes + p.u_bytes + p.raw_bytes + p.pe_bytes;
-    p.cst_bytes = (mode == CMODE_W) ? 0 : (((uint32_t)BM * k * 2 + 1023) & ~1023u);
+    p.cst_bytes = (mode == CMODE_W)
+                      ? 0
+                      : (((uint32_t)BM * k * (mode == CMODE_GF ? 4 : 2) + 1023) & ~1023u);
     p.bar_off = (uint32_t)stages * p.stage_bytes + p.cst_bytes;
     p.total = p.bar_off + 8 * (2 * stages + 5) + 16 + 1024;   // + alignment slack
     p.tx_bytes = p.a_bytes + p.u_bytes + p.pe_bytes;

@@ -46,6 +46,9 @@ _sig("sn_decompress_bwd", [_P, _ST, _P, _I64, _P, _P])
 _sig("sn_project_weight_workspace", [_P, _ST, _I64, ctypes.POINTER(_SZ)])
 _sig("sn_project_weight", [_P, _ST, _P, _I64, _I64, _I64, _P, _P, _SZ, _P])
 _sig("sn_project_weight_noalloc", [_P, _ST, _P, _I64, _I64, _I64, _P, _P])
+_sig("sn_project_tables", [_P, _ST, _P, _I64, _P, _I32, _P, _P, _P])
+_sig("sn_compress_fwd_projected", [_P, _ST, _P, _P, _P, _I64, _I32, _P, _I64, _P, _P, _P])
+_sig("sn_build_ts", [_P, _ST, _P, _I64, _P, _P, _SZ, _P])
 _sig("sn_wire_bytes", [_P, _ST, _I64, ctypes.POINTER(_SZ)])
 _sig("sn_wire_send", [_P, _P, _SZ, _P])
 _sig("sn_wire_recv", [_P, _P, _SZ, _P])
@@ -57,6 +60,7 @@ _sig("sn_status_string", [_ST], ctypes.c_char_p)
 EXPORTS = ["sn_basis_create", "sn_basis_destroy", "sn_basis_shape", "sn_compress_fwd",
            "sn_decompress_fwd", "sn_compress_bwd", "sn_decompress_bwd",
            "sn_project_weight_workspace", "sn_project_weight", "sn_project_weight_noalloc",
+           "sn_project_tables", "sn_compress_fwd_projected", "sn_build_ts",
            "sn_wire_bytes", "sn_wire_send",
            "sn_wire_recv", "sn_check_errors", "sn_launch_count", "sn_status_string"]
 
@@ -165,6 +169,71 @@ def sn_compress_fwd(basis, X, ids, tok_emb, seq_len, pos_emb=None, pos=None, out
     _check(_lib.sn_compress_fwd(basis.handle, _dtype(X), _ptr(X), _ptr(ids), _ptr(pos), T,
                                 seq_len, _ptr(tok_emb), tok_emb.shape[0], _ptr(pos_emb),
                                 _ptr(out), _stream(stream)), "sn_compress_fwd")
+    return out
+
+
+def sn_project_tables(basis, tok_emb, pos_emb=None, TU=None, PU=None, stream=None):
+    """TU = tok_emb U and PU = pos_emb U in fp32 (projected tables); returns (TU, PU)."""
+    _need(tok_emb, "tok_emb")
+    V = tok_emb.shape[0]
+    if tok_emb.shape != (V, basis.d):
+        raise ValueError("shape mismatch")
+    if TU is None:
+        TU = torch.empty(V, basis.k, dtype=torch.float32, device=tok_emb.device)
+    _need(TU, "TU", torch.float32)
+    n = 0
+    if pos_emb is not None:
+        _need(pos_emb, "pos_emb", tok_emb.dtype)
+        n = pos_emb.shape[0]
+        if pos_emb.shape != (n, basis.d):
+            raise ValueError("shape mismatch")
+        if PU is None:
+            PU = torch.empty(n, basis.k, dtype=torch.float32, device=tok_emb.device)
+        _need(PU, "PU", torch.float32)
+    else:
+        PU = None
+    _check(_lib.sn_project_tables(basis.handle, _dtype(tok_emb), _ptr(tok_emb), V, _ptr(pos_emb),
+                                  n, _ptr(TU), _ptr(PU), _stream(stream)), "sn_project_tables")
+    return TU, PU
+
+
+def sn_compress_fwd_projected(basis, X, ids, TU, seq_len, PU=None, pos=None, out=None,
+                              stream=None):
+    """C = X U - TU[ids] - PU[p]  (Eq. subtract with projected tables)."""
+    _need(X, "X")
+    _need(ids, "ids", torch.int32)
+    _need(TU, "TU", torch.float32)
+    if PU is not None:
+        _need(PU, "PU", torch.float32)
+    if pos is not None:
+        _need(pos, "pos", torch.int32)
+    T = X.shape[0]
+    if X.shape != (T, basis.d) or ids.shape != (T,) or TU.shape[1] != basis.k:
+        raise ValueError("shape mismatch")
+    if out is None:
+        out = torch.empty(T, basis.k, dtype=X.dtype, device=X.device)
+    _need(out, "out", X.dtype)
+    _check(_lib.sn_compress_fwd_projected(basis.handle, _dtype(X), _ptr(X), _ptr(ids), _ptr(pos),
+                                          T, seq_len, _ptr(TU), TU.shape[0], _ptr(PU), _ptr(out),
+                                          _stream(stream)), "sn_compress_fwd_projected")
+    return out
+
+
+def sn_build_ts(basis, tok_emb, out=None, workspace=None, stream=None):
+    """T_S = tok_emb U U^T (the low-rank token-embedding table, Sec. 4.3.1)."""
+    _need(tok_emb, "tok_emb")
+    V = tok_emb.shape[0]
+    if tok_emb.shape != (V, basis.d):
+        raise ValueError("shape mismatch")
+    if out is None:
+        out = torch.empty_like(tok_emb)
+    _need(out, "out", tok_emb.dtype)
+    nbytes = sn_wire_bytes(basis, tok_emb.dtype, V)
+    if workspace is None:
+        workspace = torch.empty(max(16, nbytes), dtype=torch.uint8, device=tok_emb.device)
+    _check(_lib.sn_build_ts(basis.handle, _dtype(tok_emb), _ptr(tok_emb), V, _ptr(out),
+                            _ptr(workspace), workspace.numel() * workspace.element_size(),
+                            _stream(stream)), "sn_build_ts")
     return out
 
 
