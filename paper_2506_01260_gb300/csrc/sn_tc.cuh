@@ -330,6 +330,14 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
     return r;
 }
 
+// Prefetch the 128-byte lines of [p, p + bytes) into L2.
+__device__ __forceinline__ void prefetch_l2_range(const void *p, int bytes)
+{
+    const uintptr_t a0 = (uintptr_t)p & ~(uintptr_t)127, a1 = (uintptr_t)p + bytes;
+    for (uintptr_t a = a0; a < a1; a += 128)
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(a));
+}
+
 // ---- cp.async: 16-byte global -> shared copies issued per thread -------------
 // Used for row gathers: each thread places its chunks directly at their
 // swizzled positions.  Completion is observed with wait_group by the issuing

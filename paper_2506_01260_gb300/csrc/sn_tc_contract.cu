@@ -205,6 +205,19 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
             const int tile = item / p.splits, split = item % p.splits;
             const int64_t r0 = MODE == CMODE_W ? (int64_t)tile * BM
                                                : tile_row0(tile, p.reorder, p.batches, p.seq_len);
+            if (MODE == CMODE_XP && r0 + row < p.rows) {
+                // this row's TU and PU rows are read after the item's main loop:
+                // start them towards L2 now (the epilogue warps are idle until then)
+                const int64_t t = r0 + row;
+                const int id = p.ids[t];
+                if (id >= 0 && id < p.vocab)
+                    prefetch_l2_range(p.TU + (int64_t)id * p.k, p.k * 4);
+                if (p.has_pe) {
+                    const int ps = p.has_pos ? p.pos[t] : (int)(t % p.seq_len);
+                    if (ps >= 0 && ps < p.seq_len)
+                        prefetch_l2_range(p.PU + (int64_t)ps * p.k, p.k * 4);
+                }
+            }
             // ---- accumulator -> output
             const uint32_t b = it & 1, nb = it >> 1;
             if (!warp_wait(accf_b + 8 * b, nb & 1, abort_flag, p.err)) {
