@@ -452,6 +452,48 @@ def run_ours(args, world, rank, local, pg):
             "note": "C = X U - (T_fixed U)[ids] - (P U)[pos] with the tables projected once "
                     "(sn_project_tables); same C as sn_compress_fwd"}}
         del TU, PU, Cp
+        # NEXT f1: the Grassmann accumulation M += G^T Cg (every iteration) and the
+        # step (every K iterations), at the workload's G and U
+        Mg = torch.zeros(d, k, dtype=torch.float32, device=dev)
+        wsa, wss = sn.sn_grassmann_workspace(basis, T)
+        wsa = torch.empty(max(256, wsa), dtype=torch.uint8, device=dev)
+        wss = torch.empty(max(256, wss), dtype=torch.uint8, device=dev)
+        sn.sn_compress_bwd(basis, G, out=Cg)
+        for _ in range(args.warmup):
+            flush.zero_()
+            sn.sn_grassmann_accumulate(basis, G, Cg, Mg, workspace=wsa)
+        gev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(min(args.steps, 30))]
+        for a_, b_ in gev:
+            flush.zero_()
+            a_.record(stream)
+            sn.sn_grassmann_accumulate(basis, G, Cg, Mg, workspace=wsa)
+            b_.record(stream)
+        torch.cuda.synchronize()
+        gms = max_over_ranks(pg, statistics.mean(a_.elapsed_time(b_) for a_, b_ in gev), dev)
+        Unew = torch.empty(d, k, dtype=torch.float32, device=dev)
+        Mg.div_(len(gev) + args.warmup)
+        sn.sn_grassmann_step(basis, Mg, 1, 1e-3, out=Unew, workspace=wss)
+        sev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(5)]
+        for a_, b_ in sev:
+            a_.record(stream)
+            sn.sn_grassmann_step(basis, Mg, 1, 1e-3, out=Unew, workspace=wss)
+            b_.record(stream)
+        torch.cuda.synchronize()
+        sn.sn_check_errors(basis)
+        sms_ = statistics.mean(a_.elapsed_time(b_) for a_, b_ in sev)
+        orth = float((Unew.double().t() @ Unew.double() - torch.eye(k, dtype=torch.float64,
+                                                                      device=dev)).abs().max())
+        gab = 2 * T * d + 2 * T * k + 2 * 4 * d * k
+        nxt["f1_grassmann"] = {
+            "accumulate_ms": gms, "accumulate_algorithmic_bytes": gab,
+            "accumulate_gbs": gab / (gms / 1e3) / 1e9,
+            "accumulate_frac": gab / (gms / 1e3) / 1e9 / hbm,
+            "step_ms": sms_, "step_orthonormality_error": orth,
+            "note": "M += G^T (G U) per iteration on the tensor cores (the [d, d] S is never "
+                    "formed); every K iterations: tangent step + CholeskyQR2 retraction"}
+        del Mg, wsa, wss, Unew
 
     # ---- end to end through the C ABI with host buffers ----
     e2e_line = None

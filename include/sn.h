@@ -50,7 +50,8 @@ typedef enum {
     SN_ERR_UNSUPPORTED = 3,   /* valid request this build does not implement */
     SN_ERR_BAD_ID = 4,        /* asynchronous: an id or position was out of range */
     SN_ERR_TIMEOUT = 5,       /* asynchronous: a bounded in-kernel wait expired */
-    SN_ERR_CUDA = 6           /* a CUDA runtime call failed */
+    SN_ERR_CUDA = 6,          /* a CUDA runtime call failed */
+    SN_ERR_NUMERIC = 7        /* asynchronous: a factorisation met a non-positive pivot */
 } sn_status;
 
 typedef enum { SN_BF16 = 0, SN_F32 = 1 } sn_dtype;
@@ -170,6 +171,43 @@ sn_status sn_compress_fwd_projected(sn_basis_t basis, sn_dtype dtype, const void
  * T_S may not overlap tok_emb or the workspace. */
 sn_status sn_build_ts(sn_basis_t basis, sn_dtype dtype, const void *tok_emb, int64_t vocab,
                       void *T_S, void *workspace, size_t workspace_bytes, sn_stream_t stream);
+
+/* ---- Subspace update on the Grassmann manifold (Sec. 4.5; gradient of Sec. 6)
+ * The Grassmann loss (1/K) sum_t ||G_t (I - U U^T)||_F^2 over the activation
+ * gradients G_t of the last compressed layer has the Euclidean gradient -2 S U
+ * with S = (1/K) sum_t G_t^T G_t.  U changes only at a step, so S U is
+ * accumulated directly as M = sum_t G_t^T (G_t U) = K S U: G_t U is the
+ * compressed gradient Cg of Eq. (grad_compress) (sn_compress_bwd), and the
+ * [d, d] matrix S is never formed.  Every K iterations the step takes the
+ * tangent component of -2 M / K, moves U by -eta times it and retracts onto the
+ * manifold with a QR factorisation (diag(R) > 0); a new basis handle is then
+ * created from the result. */
+
+/* Workspace bytes of sn_grassmann_accumulate for T tokens and of
+ * sn_grassmann_step (either pointer may be NULL). */
+sn_status sn_grassmann_workspace(sn_basis_t basis, int64_t T, size_t *accumulate_bytes,
+                                 size_t *step_bytes);
+
+/* M += G^T Cg.  G: bf16 [T, d]; Cg: bf16 [T, k] = G U from sn_compress_bwd with
+ * this basis; M: fp32 [d, k] row-major, caller-owned (zero it at the start of a
+ * window of K iterations).  Accumulated on the tensor cores in fp32.  bf16 only. */
+sn_status sn_grassmann_accumulate(sn_basis_t basis, sn_dtype dtype, const void *G, const void *Cg,
+                                  int64_t T, float *M, void *workspace, size_t workspace_bytes,
+                                  sn_stream_t stream);
+
+/* *acc += ||G (I - U U^T)||_F^2, evaluated as ||G||_F^2 - ||Cg||_F^2 in fp64 from
+ * the bf16 tensors (so its error is ~2^-8 ||G||_F^2: a monitoring metric for
+ * gradients that are not almost entirely inside the subspace).  acc: device
+ * fp64 scalar.  bf16 only. */
+sn_status sn_grassmann_residual(sn_basis_t basis, sn_dtype dtype, const void *G, const void *Cg,
+                                int64_t T, double *acc, sn_stream_t stream);
+
+/* U_new = Q of U - eta * tangent(-2 M / K), the QR factor with diag(R) > 0
+ * (CholeskyQR2 with fp64 Gram matrices).  M: fp32 [d, k] from
+ * sn_grassmann_accumulate over K >= 1 iterations; U_new: fp32 [d, k], may not
+ * overlap M.  A non-positive pivot records SN_ERR_NUMERIC for sn_check_errors. */
+sn_status sn_grassmann_step(sn_basis_t basis, const float *M, int32_t K, float eta, float *U_new,
+                            void *workspace, size_t workspace_bytes, sn_stream_t stream);
 
 /* Bytes on the wire for T tokens: T * k * element size (Sec. 4.3: k/d of X). */
 sn_status sn_wire_bytes(sn_basis_t basis, sn_dtype dtype, int64_t T, size_t *bytes);

@@ -79,6 +79,7 @@ const char *sn_status_string(sn_status s)
     case SN_ERR_BAD_ID: return "SN_ERR_BAD_ID";
     case SN_ERR_TIMEOUT: return "SN_ERR_TIMEOUT";
     case SN_ERR_CUDA: return "SN_ERR_CUDA";
+    case SN_ERR_NUMERIC: return "SN_ERR_NUMERIC";
     }
     return "SN_ERR_UNKNOWN";
 }
@@ -348,6 +349,86 @@ sn_status sn_build_ts(sn_basis_t b, sn_dtype dt, const void *tok, int64_t vocab,
     return cuda_status(e);
 }
 
+sn_status sn_grassmann_workspace(sn_basis_t b, int64_t T, size_t *acc_bytes, size_t *step_bytes)
+{
+    sn_status st = check_basis(b, SN_BF16);
+    if (st != SN_OK)
+        return st;
+    if (T < 0 || T >= kMaxRows)
+        return SN_ERR_INVALID_ARG;
+    if (acc_bytes)
+        *acc_bytes = sn::tc_grassmann_workspace(*b, T > 0 ? T : 1);
+    if (step_bytes)
+        *step_bytes = sn::grassmann_step_workspace(*b);
+    return SN_OK;
+}
+
+sn_status sn_grassmann_accumulate(sn_basis_t b, sn_dtype dt, const void *G, const void *Cg,
+                                  int64_t T, float *M, void *ws, size_t ws_bytes,
+                                  sn_stream_t stream)
+{
+    sn_status st = check_basis(b, dt);
+    if (st != SN_OK)
+        return st;
+    if (dt != SN_BF16)
+        return SN_ERR_UNSUPPORTED;
+    if (T < 0 || T >= kMaxRows)
+        return SN_ERR_INVALID_ARG;
+    if (T == 0)
+        return SN_OK;
+    if (!G || !Cg || !M || !ws || ws_bytes < sn::tc_grassmann_workspace(*b, T))
+        return SN_ERR_INVALID_ARG;
+    if (!aligned(G, 16) || !aligned(Cg, 16) || !aligned(M, 16) || !aligned(ws, 256))
+        return SN_ERR_ALIGNMENT;
+    const size_t mb = (size_t)b->d * b->k * 4;
+    if (overlap(M, mb, G, (size_t)T * b->d * 2) || overlap(M, mb, Cg, (size_t)T * b->k * 2) ||
+        overlap(ws, ws_bytes, M, mb) || overlap(ws, ws_bytes, G, (size_t)T * b->d * 2) ||
+        overlap(ws, ws_bytes, Cg, (size_t)T * b->k * 2))
+        return SN_ERR_INVALID_ARG;
+    return cuda_status(sn::tc_grassmann_accumulate(*b, (const __nv_bfloat16 *)G,
+                                                   (const __nv_bfloat16 *)Cg, T, M, ws,
+                                                   (cudaStream_t)stream));
+}
+
+sn_status sn_grassmann_residual(sn_basis_t b, sn_dtype dt, const void *G, const void *Cg,
+                                int64_t T, double *acc, sn_stream_t stream)
+{
+    sn_status st = check_basis(b, dt);
+    if (st != SN_OK)
+        return st;
+    if (dt != SN_BF16)
+        return SN_ERR_UNSUPPORTED;
+    if (T < 0 || T >= kMaxRows || !acc)
+        return SN_ERR_INVALID_ARG;
+    if (T == 0)
+        return SN_OK;
+    if (!G || !Cg)
+        return SN_ERR_INVALID_ARG;
+    if (!aligned(G, 16) || !aligned(Cg, 2) || !aligned(acc, 8))
+        return SN_ERR_ALIGNMENT;
+    return cuda_status(sn::grassmann_residual(*b, (const __nv_bfloat16 *)G,
+                                              (const __nv_bfloat16 *)Cg, T, acc,
+                                              (cudaStream_t)stream));
+}
+
+sn_status sn_grassmann_step(sn_basis_t b, const float *M, int32_t K, float eta, float *U_new,
+                            void *ws, size_t ws_bytes, sn_stream_t stream)
+{
+    sn_status st = check_basis(b, SN_F32);
+    if (st != SN_OK)
+        return st;
+    if (!M || !U_new || !ws || K < 1 || !(eta >= 0.f) ||
+        ws_bytes < sn::grassmann_step_workspace(*b))
+        return SN_ERR_INVALID_ARG;
+    if (!aligned(M, 16) || !aligned(U_new, 16) || !aligned(ws, 256))
+        return SN_ERR_ALIGNMENT;
+    const size_t mb = (size_t)b->d * b->k * 4;
+    if (overlap(M, mb, U_new, mb) || overlap(ws, ws_bytes, M, mb) ||
+        overlap(ws, ws_bytes, U_new, mb))
+        return SN_ERR_INVALID_ARG;
+    return cuda_status(sn::grassmann_step(*b, M, K, eta, U_new, ws, (cudaStream_t)stream));
+}
+
 sn_status sn_wire_bytes(sn_basis_t b, sn_dtype dt, int64_t T, size_t *bytes)
 {
     if (!b || !bytes || T < 0 || (dt != SN_BF16 && dt != SN_F32))
@@ -392,6 +473,8 @@ sn_status sn_check_errors(sn_basis_t b, sn_stream_t stream)
         return SN_ERR_TIMEOUT;
     if (word & SN_EBIT_BAD_ID)
         return SN_ERR_BAD_ID;
+    if (word & SN_EBIT_NUMERIC)
+        return SN_ERR_NUMERIC;
     return SN_OK;
 }
 

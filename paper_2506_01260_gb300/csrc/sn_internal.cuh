@@ -11,6 +11,7 @@
 enum : unsigned int {
     SN_EBIT_BAD_ID = 1u,    // an id or position was out of range (row zeroed)
     SN_EBIT_TIMEOUT = 2u,   // a bounded wait expired; the kernel gave up
+    SN_EBIT_NUMERIC = 4u,   // a factorisation met a non-positive pivot
 };
 
 // Padded copies of U kept by a basis handle.
@@ -72,6 +73,17 @@ size_t tc_project_workspace(const sn_basis &b, int64_t cols);
 // out[r, :] = A[r, :] U in fp32 (projected tables: T_fixed U, P U)
 cudaError_t tc_contract_f32(const sn_basis &b, const __nv_bfloat16 *A, int64_t rows, float *out,
                             cudaStream_t s);
+// Grassmann accumulation M += G^T Cg (M fp32 [d, k]); workspace bytes for T tokens
+size_t tc_grassmann_workspace(const sn_basis &b, int64_t T);
+cudaError_t tc_grassmann_accumulate(const sn_basis &b, const __nv_bfloat16 *G,
+                                    const __nv_bfloat16 *Cg, int64_t T, float *M, void *workspace,
+                                    cudaStream_t s);
+// ||G||^2 - ||Cg||^2 added to *acc (fp64); the Grassmann step (CUDA cores)
+cudaError_t grassmann_residual(const sn_basis &b, const __nv_bfloat16 *G,
+                               const __nv_bfloat16 *Cg, int64_t T, double *acc, cudaStream_t s);
+size_t grassmann_step_workspace(const sn_basis &b);
+cudaError_t grassmann_step(const sn_basis &b, const float *M, int K, float eta, float *U_new,
+                           void *workspace, cudaStream_t s);
 // C = X U - TU[ids] - PU[pos] (PU may be null)
 cudaError_t tc_compress_projected(const sn_basis &b, const __nv_bfloat16 *X, const int32_t *ids,
                                   const int32_t *pos, int64_t T, int seq_len, const float *TU,

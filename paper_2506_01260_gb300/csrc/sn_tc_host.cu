@@ -2,6 +2,7 @@
 // shared-memory stage planning, work splitting, and the launch sequences of
 // the boundary calls.
 #include <algorithm>
+#include <climits>
 #include <cstring>
 #include <mutex>
 
@@ -338,6 +339,101 @@ size_t tc_project_workspace(const sn_basis &b, int64_t cols)
     project_splits(b.d, cols, sm_count(current_device()), &splits, &kc_per);
     return align256(sizeof(float) * (size_t)splits * cols * b.n_pad) +
            align256(sizeof(__nv_bfloat16) * (size_t)cols * b.k64);
+}
+
+namespace tc {
+namespace {
+
+// CgT[j, t] = Cg[t, j] for j < k, t < T; zero for k <= j < n_pad and T <= t < Tp.
+__global__ void k_transpose_pad(const __nv_bfloat16 *__restrict__ Cg, int64_t T, int k, int n_pad,
+                                int64_t Tp, __nv_bfloat16 *__restrict__ CgT)
+{
+    const int64_t n = (int64_t)n_pad * Tp;
+    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n;
+         e += (int64_t)gridDim.x * blockDim.x) {
+        const int j = (int)(e / Tp);
+        const int64_t t = e - (int64_t)j * Tp;
+        CgT[e] = (j < k && t < T) ? Cg[t * k + j] : __float2bfloat16_rn(0.f);
+    }
+}
+
+// M[i, j] += sum over splits of P[split, i, j], j < k (M row-major [d, k]).
+__global__ void k_accumulate_partials(const float *__restrict__ P, int splits, int64_t d,
+                                      int n_pad, int k, float *__restrict__ M)
+{
+    const int64_t n = d * k;
+    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n;
+         e += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t i = e / k;
+        const int j = (int)(e - i * k);
+        float s = 0.f;
+        for (int sp = 0; sp < splits; ++sp)
+            s += __ldg(P + ((int64_t)sp * d + i) * n_pad + j);
+        M[e] += s;
+    }
+}
+
+}  // namespace
+}  // namespace tc
+
+size_t tc_grassmann_workspace(const sn_basis &b, int64_t T)
+{
+    using namespace tc;
+    int splits, kc_per;
+    project_splits((int)std::min<int64_t>(T, INT32_MAX), b.d, sm_count(current_device()), &splits,
+                   &kc_per);
+    const int64_t Tp = (T + 63) / 64 * 64;
+    return align256(sizeof(__nv_bfloat16) * (size_t)b.n_pad * Tp) +
+           align256(sizeof(float) * (size_t)splits * b.d * b.n_pad);
+}
+
+cudaError_t tc_grassmann_accumulate(const sn_basis &b, const __nv_bfloat16 *G,
+                                    const __nv_bfloat16 *Cg, int64_t T, float *M, void *workspace,
+                                    cudaStream_t s)
+{
+    using namespace tc;
+    const int sms = sm_count(current_device());
+    int splits, kc_per;
+    project_splits((int)T, b.d, sms, &splits, &kc_per);
+    const int64_t Tp = (T + 63) / 64 * 64;
+    __nv_bfloat16 *CgT = (__nv_bfloat16 *)workspace;
+    float *P = (float *)((char *)workspace +
+                         align256(sizeof(__nv_bfloat16) * (size_t)b.n_pad * Tp));
+    // Cg^T, K-major over the tokens: the B operand of M = G^T Cg
+    k_transpose_pad<<<4 * sms, 256, 0, s>>>(Cg, T, b.k, b.n_pad, Tp, CgT);
+    count_launch();
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess)
+        return e;
+    // fp32 partials of G^T Cg over token ranges: the projection's first pass with G
+    // in the role of W (read MN-major) and Cg^T in the role of U^T
+    ContractParams p;
+    std::memset(&p, 0, sizeof p);
+    bool ok = map2d(&p.mapA, G, b.d, T, (uint64_t)b.d * 2, 64, BK, true) &&
+              map2d(&p.mapU, CgT, Tp, b.n_pad, (uint64_t)Tp * 2, BK, b.n_pad, true);
+    p.mapPE = p.mapA;
+    if (!ok)
+        return cudaErrorInvalidValue;
+    p.P = P;
+    p.err = b.err;
+    p.rows = b.d;
+    p.vocab = 1;
+    p.seq_len = 1;
+    p.d = (int)T;
+    p.k = b.k;
+    p.n_pad = b.n_pad;
+    p.acc_stride = pow2_at_least(b.n_pad, 32);
+    p.nkc = (int)((T + BK - 1) / BK);
+    p.kc_per_item = kc_per;
+    p.splits = splits;
+    p.ntiles = (b.d + BM - 1) / BM;
+    p.stages = contract_stages(CMODE_W, b.n_pad, b.k, 0);
+    e = launch_contract(CMODE_W, p, std::min(p.ntiles * splits, sms), s);
+    if (e != cudaSuccess)
+        return e;
+    k_accumulate_partials<<<4 * sms, 256, 0, s>>>(P, splits, b.d, b.n_pad, b.k, M);
+    count_launch();
+    return cudaGetLastError();
 }
 
 cudaError_t tc_project(const sn_basis &b, const __nv_bfloat16 *W, int64_t cols, int64_t ld,

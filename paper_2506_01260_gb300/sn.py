@@ -16,7 +16,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libsn.so")
 
 SN_OK, SN_ERR_INVALID_ARG, SN_ERR_ALIGNMENT, SN_ERR_UNSUPPORTED = 0, 1, 2, 3
-SN_ERR_BAD_ID, SN_ERR_TIMEOUT, SN_ERR_CUDA = 4, 5, 6
+SN_ERR_BAD_ID, SN_ERR_TIMEOUT, SN_ERR_CUDA, SN_ERR_NUMERIC = 4, 5, 6, 7
 SN_BF16, SN_F32 = 0, 1
 
 if not os.path.exists(LIB_PATH):
@@ -49,6 +49,10 @@ _sig("sn_project_weight_noalloc", [_P, _ST, _P, _I64, _I64, _I64, _P, _P])
 _sig("sn_project_tables", [_P, _ST, _P, _I64, _P, _I32, _P, _P, _P])
 _sig("sn_compress_fwd_projected", [_P, _ST, _P, _P, _P, _I64, _I32, _P, _I64, _P, _P, _P])
 _sig("sn_build_ts", [_P, _ST, _P, _I64, _P, _P, _SZ, _P])
+_sig("sn_grassmann_workspace", [_P, _I64, ctypes.POINTER(_SZ), ctypes.POINTER(_SZ)])
+_sig("sn_grassmann_accumulate", [_P, _ST, _P, _P, _I64, _P, _P, _SZ, _P])
+_sig("sn_grassmann_residual", [_P, _ST, _P, _P, _I64, _P, _P])
+_sig("sn_grassmann_step", [_P, _P, _I32, ctypes.c_float, _P, _P, _SZ, _P])
 _sig("sn_wire_bytes", [_P, _ST, _I64, ctypes.POINTER(_SZ)])
 _sig("sn_wire_send", [_P, _P, _SZ, _P])
 _sig("sn_wire_recv", [_P, _P, _SZ, _P])
@@ -61,6 +65,8 @@ EXPORTS = ["sn_basis_create", "sn_basis_destroy", "sn_basis_shape", "sn_compress
            "sn_decompress_fwd", "sn_compress_bwd", "sn_decompress_bwd",
            "sn_project_weight_workspace", "sn_project_weight", "sn_project_weight_noalloc",
            "sn_project_tables", "sn_compress_fwd_projected", "sn_build_ts",
+           "sn_grassmann_workspace", "sn_grassmann_accumulate", "sn_grassmann_residual",
+           "sn_grassmann_step",
            "sn_wire_bytes", "sn_wire_send",
            "sn_wire_recv", "sn_check_errors", "sn_launch_count", "sn_status_string"]
 
@@ -234,6 +240,61 @@ def sn_build_ts(basis, tok_emb, out=None, workspace=None, stream=None):
     _check(_lib.sn_build_ts(basis.handle, _dtype(tok_emb), _ptr(tok_emb), V, _ptr(out),
                             _ptr(workspace), workspace.numel() * workspace.element_size(),
                             _stream(stream)), "sn_build_ts")
+    return out
+
+
+def sn_grassmann_workspace(basis, T):
+    """(accumulate bytes for T tokens, step bytes)."""
+    a, b = _SZ(), _SZ()
+    _check(_lib.sn_grassmann_workspace(basis.handle, T, ctypes.byref(a), ctypes.byref(b)),
+           "sn_grassmann_workspace")
+    return int(a.value), int(b.value)
+
+
+def sn_grassmann_accumulate(basis, G, Cg, M, workspace=None, stream=None):
+    """M += G^T Cg (Cg = G U from sn_compress_bwd); M fp32 [d, k] (Sec. 4.5, Sec. 6)."""
+    _need(G, "G", torch.bfloat16)
+    _need(Cg, "Cg", torch.bfloat16)
+    _need(M, "M", torch.float32)
+    T = G.shape[0]
+    if G.shape != (T, basis.d) or Cg.shape != (T, basis.k) or M.shape != (basis.d, basis.k):
+        raise ValueError("shape mismatch")
+    if workspace is None:
+        workspace = torch.empty(max(256, sn_grassmann_workspace(basis, T)[0]), dtype=torch.uint8,
+                                device=G.device)
+    _check(_lib.sn_grassmann_accumulate(basis.handle, SN_BF16, _ptr(G), _ptr(Cg), T, _ptr(M),
+                                        _ptr(workspace), workspace.numel(), _stream(stream)),
+           "sn_grassmann_accumulate")
+    return M
+
+
+def sn_grassmann_residual(basis, G, Cg, acc, stream=None):
+    """acc (device fp64 scalar) += ||G (I - U U^T)||_F^2 = ||G||^2 - ||Cg||^2."""
+    _need(G, "G", torch.bfloat16)
+    _need(Cg, "Cg", torch.bfloat16)
+    _need(acc, "acc", torch.float64)
+    T = G.shape[0]
+    if G.shape != (T, basis.d) or Cg.shape != (T, basis.k) or acc.numel() < 1:
+        raise ValueError("shape mismatch")
+    _check(_lib.sn_grassmann_residual(basis.handle, SN_BF16, _ptr(G), _ptr(Cg), T, _ptr(acc),
+                                      _stream(stream)), "sn_grassmann_residual")
+    return acc
+
+
+def sn_grassmann_step(basis, M, K, eta, out=None, workspace=None, stream=None):
+    """U_new = QR-retraction of U - eta * tangent(-2 M / K) (Sec. 4.5); fp32 [d, k]."""
+    _need(M, "M", torch.float32)
+    if M.shape != (basis.d, basis.k):
+        raise ValueError("shape mismatch")
+    if out is None:
+        out = torch.empty_like(M)
+    _need(out, "out", torch.float32)
+    if workspace is None:
+        workspace = torch.empty(max(256, sn_grassmann_workspace(basis, 1)[1]), dtype=torch.uint8,
+                                device=M.device)
+    _check(_lib.sn_grassmann_step(basis.handle, _ptr(M), int(K), float(eta), _ptr(out),
+                                  _ptr(workspace), workspace.numel(), _stream(stream)),
+           "sn_grassmann_step")
     return out
 
 
