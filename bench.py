@@ -494,6 +494,33 @@ def run_ours(args, world, rank, local, pg):
             "note": "M += G^T (G U) per iteration on the tensor cores (the [d, d] S is never "
                     "formed); every K iterations: tangent step + CholeskyQR2 retraction"}
         del Mg, wsa, wss, Unew
+        # NEXT f2: one row-constant AdamW step on an fp32 master copy of W_o
+        # (bf16 gradient), the weight whose columns the paper keeps in S
+        Wm = Wo.float()
+        gW = (0.01 * torch.randn(wo_shape, generator=g, device=dev)).to(torch.bfloat16)
+        Mm = torch.zeros_like(Wm)
+        Vm = torch.zeros_like(Wm)
+        aws = torch.empty(wo_shape[1], dtype=torch.float32, device=dev)
+        for t_ in range(1, args.warmup + 1):
+            flush.zero_()
+            sn.sn_adamw_rowconst(Wm, gW, Mm, Vm, t_, 1e-4, workspace=aws)
+        aev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(min(args.steps, 30))]
+        for i_, (a_, b_) in enumerate(aev):
+            flush.zero_()
+            a_.record(stream)
+            sn.sn_adamw_rowconst(Wm, gW, Mm, Vm, args.warmup + 1 + i_, 1e-4, workspace=aws)
+            b_.record(stream)
+        torch.cuda.synchronize()
+        ams = max_over_ranks(pg, statistics.mean(a_.elapsed_time(b_) for a_, b_ in aev), dev)
+        nel = wo_shape[0] * wo_shape[1]
+        aab = nel * (2 + 8 + 8 + 8)
+        nxt["f2_adamw_rowconst"] = {
+            "ms": ams, "algorithmic_bytes": aab, "gbs": aab / (ams / 1e3) / 1e9,
+            "frac": aab / (ams / 1e3) / 1e9 / hbm, "shape": list(wo_shape),
+            "note": "fp32 W, M, V, bf16 gradient; moments + column sums of V^ (pass 1), "
+                    "W update with one rate per column (pass 2, re-reads M)"}
+        del Wm, gW, Mm, Vm, aws
 
     # ---- end to end through the C ABI with host buffers ----
     e2e_line = None

@@ -209,6 +209,26 @@ sn_status sn_grassmann_residual(sn_basis_t basis, sn_dtype dtype, const void *G,
 sn_status sn_grassmann_step(sn_basis_t basis, const float *M, int32_t K, float eta, float *U_new,
                             void *workspace, size_t workspace_bytes, sn_stream_t stream);
 
+/* ---- Row-constant AdamW for W_p2 (Sec. 5) ---------------------------------------
+ * Element-wise AdamW rescales each coordinate of an update by its own rate,
+ * which turns rows of the update out of S.  The paper keeps one adaptive rate
+ * per row of W_p2 (the mean of the bias-corrected second moment over the row),
+ * so a weight whose rows lie in S stays there under in-S gradients without
+ * further projection.  In the torch layout W is [rows = d, cols = d_ff] and the
+ * paper's rows are its columns: one rate per column.  One step t >= 1:
+ *   M = beta1 M + (1 - beta1) g,  V = beta2 V + (1 - beta2) g^2
+ *   W = W - lr (M / (1 - beta1^t)) / (sqrt(mean_col(V) / (1 - beta2^t)) + eps) - lambda W
+ * (the bias correction is AdamW's 1 - beta^t; the paper's printed V/(beta2 + eps)
+ * is read as that; lambda is applied as printed, i.e. torch's lr * weight_decay).
+ * W, M, V: fp32 [rows, cols], updated in place (zero M and V before step 1);
+ * grad: [rows, cols] in `grad_dtype` (SN_BF16 or SN_F32); workspace: device
+ * memory of at least cols * 4 bytes, used only during the call.  No basis is
+ * involved.  Buffers may not overlap. */
+sn_status sn_adamw_rowconst(sn_dtype grad_dtype, float *W, const void *grad, float *M, float *V,
+                            int64_t rows, int64_t cols, int64_t step, float lr, float beta1,
+                            float beta2, float eps, float lambda, void *workspace,
+                            size_t workspace_bytes, sn_stream_t stream);
+
 /* Bytes on the wire for T tokens: T * k * element size (Sec. 4.3: k/d of X). */
 sn_status sn_wire_bytes(sn_basis_t basis, sn_dtype dtype, int64_t T, size_t *bytes);
 

@@ -429,6 +429,30 @@ sn_status sn_grassmann_step(sn_basis_t b, const float *M, int32_t K, float eta, 
     return cuda_status(sn::grassmann_step(*b, M, K, eta, U_new, ws, (cudaStream_t)stream));
 }
 
+sn_status sn_adamw_rowconst(sn_dtype gdt, float *W, const void *g, float *M, float *V,
+                            int64_t rows, int64_t cols, int64_t t, float lr, float b1, float b2,
+                            float eps, float lam, void *ws, size_t ws_bytes, sn_stream_t stream)
+{
+    if (gdt != SN_BF16 && gdt != SN_F32)
+        return SN_ERR_INVALID_ARG;
+    if (rows <= 0 || cols <= 0 || rows >= kMaxRows || cols >= kMaxRows || t < 1 ||
+        !(b1 >= 0.f && b1 < 1.f) || !(b2 >= 0.f && b2 < 1.f) || !(eps >= 0.f) || !(lr >= 0.f) ||
+        !(lam >= 0.f) || !W || !g || !M || !V || !ws || ws_bytes < (size_t)cols * 4)
+        return SN_ERR_INVALID_ARG;
+    if (!aligned(W, 16) || !aligned(g, 16) || !aligned(M, 16) || !aligned(V, 16) ||
+        !aligned(ws, 16))
+        return SN_ERR_ALIGNMENT;
+    const size_t n4 = (size_t)rows * cols * 4, ng = (size_t)rows * cols * esize(gdt);
+    const void *bufs[5] = {W, g, M, V, ws};
+    const size_t lens[5] = {n4, ng, n4, n4, (size_t)cols * 4};
+    for (int i = 0; i < 5; ++i)
+        for (int j = i + 1; j < 5; ++j)
+            if (overlap(bufs[i], lens[i], bufs[j], lens[j]))
+                return SN_ERR_INVALID_ARG;
+    return cuda_status(sn::adamw_rowconst(gdt == SN_BF16, W, g, M, V, rows, cols, t, lr, b1, b2,
+                                          eps, lam, (float *)ws, (cudaStream_t)stream));
+}
+
 sn_status sn_wire_bytes(sn_basis_t b, sn_dtype dt, int64_t T, size_t *bytes)
 {
     if (!b || !bytes || T < 0 || (dt != SN_BF16 && dt != SN_F32))

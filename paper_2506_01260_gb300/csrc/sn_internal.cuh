@@ -84,6 +84,10 @@ cudaError_t grassmann_residual(const sn_basis &b, const __nv_bfloat16 *G,
 size_t grassmann_step_workspace(const sn_basis &b);
 cudaError_t grassmann_step(const sn_basis &b, const float *M, int K, float eta, float *U_new,
                            void *workspace, cudaStream_t s);
+// Row-constant AdamW step (fp32 W, M, V; grad bf16 or fp32); colsum: [cols] fp32 scratch
+cudaError_t adamw_rowconst(bool grad_bf16, float *W, const void *g, float *M, float *V,
+                           int64_t rows, int64_t cols, int64_t t, float lr, float b1, float b2,
+                           float eps, float lam, float *colsum, cudaStream_t s);
 // C = X U - TU[ids] - PU[pos] (PU may be null)
 cudaError_t tc_compress_projected(const sn_basis &b, const __nv_bfloat16 *X, const int32_t *ids,
                                   const int32_t *pos, int64_t T, int seq_len, const float *TU,

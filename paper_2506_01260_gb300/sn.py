@@ -53,6 +53,8 @@ _sig("sn_grassmann_workspace", [_P, _I64, ctypes.POINTER(_SZ), ctypes.POINTER(_S
 _sig("sn_grassmann_accumulate", [_P, _ST, _P, _P, _I64, _P, _P, _SZ, _P])
 _sig("sn_grassmann_residual", [_P, _ST, _P, _P, _I64, _P, _P])
 _sig("sn_grassmann_step", [_P, _P, _I32, ctypes.c_float, _P, _P, _SZ, _P])
+_sig("sn_adamw_rowconst", [_ST, _P, _P, _P, _P, _I64, _I64, _I64, ctypes.c_float, ctypes.c_float,
+                           ctypes.c_float, ctypes.c_float, ctypes.c_float, _P, _SZ, _P])
 _sig("sn_wire_bytes", [_P, _ST, _I64, ctypes.POINTER(_SZ)])
 _sig("sn_wire_send", [_P, _P, _SZ, _P])
 _sig("sn_wire_recv", [_P, _P, _SZ, _P])
@@ -66,7 +68,7 @@ EXPORTS = ["sn_basis_create", "sn_basis_destroy", "sn_basis_shape", "sn_compress
            "sn_project_weight_workspace", "sn_project_weight", "sn_project_weight_noalloc",
            "sn_project_tables", "sn_compress_fwd_projected", "sn_build_ts",
            "sn_grassmann_workspace", "sn_grassmann_accumulate", "sn_grassmann_residual",
-           "sn_grassmann_step",
+           "sn_grassmann_step", "sn_adamw_rowconst",
            "sn_wire_bytes", "sn_wire_send",
            "sn_wire_recv", "sn_check_errors", "sn_launch_count", "sn_status_string"]
 
@@ -296,6 +298,26 @@ def sn_grassmann_step(basis, M, K, eta, out=None, workspace=None, stream=None):
                                   _ptr(workspace), workspace.numel(), _stream(stream)),
            "sn_grassmann_step")
     return out
+
+
+def sn_adamw_rowconst(W, grad, M, V, step, lr, beta1=0.9, beta2=0.999, eps=1e-8, lam=0.0,
+                      workspace=None, stream=None):
+    """One row-constant AdamW step on W [d, cols] (one adaptive rate per column; Sec. 5).
+    W, M, V fp32, updated in place; grad bf16 or fp32."""
+    for t_, nm in ((W, "W"), (M, "M"), (V, "V")):
+        _need(t_, nm, torch.float32)
+    _need(grad, "grad")
+    if W.dim() != 2 or grad.shape != W.shape or M.shape != W.shape or V.shape != W.shape:
+        raise ValueError("shape mismatch")
+    rows, cols = W.shape
+    if workspace is None:
+        workspace = torch.empty(cols, dtype=torch.float32, device=W.device)
+    _check(_lib.sn_adamw_rowconst(_dtype(grad), _ptr(W), _ptr(grad), _ptr(M), _ptr(V), rows, cols,
+                                  int(step), float(lr), float(beta1), float(beta2), float(eps),
+                                  float(lam), _ptr(workspace),
+                                  workspace.numel() * workspace.element_size(), _stream(stream)),
+           "sn_adamw_rowconst")
+    return W
 
 
 def sn_decompress_fwd(basis, C, ids, tok_emb, seq_len, pos_emb=None, pos=None, out=None,
