@@ -472,6 +472,8 @@ def run_ours(args, world, rank, local, pg):
         torch.cuda.synchronize()
         gms = max_over_ranks(pg, statistics.mean(a_.elapsed_time(b_) for a_, b_ in gev), dev)
         Unew = torch.empty(d, k, dtype=torch.float32, device=dev)
+        from paper_2506_01260_gb300.shard import allreduce_grassmann
+        allreduce_grassmann(Mg)        # data-parallel replicas sum M before the step
         Mg.div_(len(gev) + args.warmup)
         sn.sn_grassmann_step(basis, Mg, 1, 1e-3, out=Unew, workspace=wss)
         sev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
