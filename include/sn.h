@@ -229,6 +229,32 @@ sn_status sn_adamw_rowconst(sn_dtype grad_dtype, float *W, const void *grad, flo
                             float beta2, float eps, float lambda, void *workspace,
                             size_t workspace_bytes, sn_stream_t stream);
 
+/* ---- Lossy comparators (Sec. 8, comparison against lossy compressions) --------
+ * What a stage boundary could send instead of C at (about) the same number of
+ * bytes, for measuring their reconstruction error on the same batches.  X is a
+ * bf16 batch [T, d] with d % 8 == 0; everything is device memory.  bf16 only. */
+
+/* Per row, the kk entries of largest magnitude (ties towards the lower column)
+ * in ascending column order: values bf16 [T, kk], cols uint16 [T, kk].
+ * 1 <= kk <= min(d, 4096), d <= 65536.  At 4 bytes per kept entry, kk = k / 2
+ * matches the subspace codec's 2 k bytes per token. */
+sn_status sn_topk_compress(const void *X, int64_t T, int32_t d, int32_t kk, void *values,
+                           uint16_t *cols, sn_stream_t stream);
+
+/* X_out [T, d] bf16: zero except values[t, j] at column cols[t, j]. */
+sn_status sn_topk_restore(const void *values, const uint16_t *cols, int64_t T, int32_t d,
+                          int32_t kk, void *X_out, sn_stream_t stream);
+
+/* One bit per entry, 1 where X < 0 (bit c % 32 of word c / 32 of the row's
+ * ceil(d / 32) words of `bits`), and scale[t] = mean |X[t, :]| (fp32): 16 times
+ * smaller than bf16, the best rate of a quantizer. */
+sn_status sn_sign_compress(const void *X, int64_t T, int32_t d, uint32_t *bits, float *scale,
+                           sn_stream_t stream);
+
+/* X_out[t, c] = -scale[t] where the bit is set, else scale[t] (bf16). */
+sn_status sn_sign_restore(const uint32_t *bits, const float *scale, int64_t T, int32_t d,
+                          void *X_out, sn_stream_t stream);
+
 /* Bytes on the wire for T tokens: T * k * element size (Sec. 4.3: k/d of X). */
 sn_status sn_wire_bytes(sn_basis_t basis, sn_dtype dtype, int64_t T, size_t *bytes);
 

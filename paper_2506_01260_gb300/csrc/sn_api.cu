@@ -453,6 +453,88 @@ sn_status sn_adamw_rowconst(sn_dtype gdt, float *W, const void *g, float *M, flo
                                           eps, lam, (float *)ws, (cudaStream_t)stream));
 }
 
+namespace {
+sn_status check_batch(const void *X, int64_t T, int32_t d)
+{
+    if (T < 0 || T >= kMaxRows || d <= 0 || d % 8 != 0 || !X)
+        return SN_ERR_INVALID_ARG;
+    return aligned(X, 16) ? SN_OK : SN_ERR_ALIGNMENT;
+}
+}  // namespace
+
+sn_status sn_topk_compress(const void *X, int64_t T, int32_t d, int32_t kk, void *vals,
+                           uint16_t *cols, sn_stream_t stream)
+{
+    sn_status st = check_batch(X, T, d);
+    if (st != SN_OK)
+        return st;
+    if (d > 65536 || kk < 1 || kk > d || kk > 4096 || !vals || !cols)
+        return SN_ERR_INVALID_ARG;
+    if (!aligned(vals, 2) || !aligned(cols, 2))
+        return SN_ERR_ALIGNMENT;
+    if (T == 0)
+        return SN_OK;
+    const size_t nx = (size_t)T * d * 2, nk = (size_t)T * kk * 2;
+    if (overlap(X, nx, vals, nk) || overlap(X, nx, cols, nk) || overlap(vals, nk, cols, nk))
+        return SN_ERR_INVALID_ARG;
+    return cuda_status(sn::lossy_topk(X, T, d, kk, vals, cols, (cudaStream_t)stream));
+}
+
+sn_status sn_topk_restore(const void *vals, const uint16_t *cols, int64_t T, int32_t d,
+                          int32_t kk, void *X_out, sn_stream_t stream)
+{
+    sn_status st = check_batch(X_out, T, d);
+    if (st != SN_OK)
+        return st;
+    if (d > 65536 || kk < 1 || kk > d || !vals || !cols)
+        return SN_ERR_INVALID_ARG;
+    if (!aligned(vals, 2) || !aligned(cols, 2))
+        return SN_ERR_ALIGNMENT;
+    if (T == 0)
+        return SN_OK;
+    const size_t nx = (size_t)T * d * 2, nk = (size_t)T * kk * 2;
+    if (overlap(X_out, nx, vals, nk) || overlap(X_out, nx, cols, nk))
+        return SN_ERR_INVALID_ARG;
+    return cuda_status(sn::lossy_topk_restore(vals, cols, T, d, kk, X_out, (cudaStream_t)stream));
+}
+
+sn_status sn_sign_compress(const void *X, int64_t T, int32_t d, uint32_t *bits, float *scale,
+                           sn_stream_t stream)
+{
+    sn_status st = check_batch(X, T, d);
+    if (st != SN_OK)
+        return st;
+    if (!bits || !scale)
+        return SN_ERR_INVALID_ARG;
+    if (!aligned(bits, 4) || !aligned(scale, 4))
+        return SN_ERR_ALIGNMENT;
+    if (T == 0)
+        return SN_OK;
+    const size_t nx = (size_t)T * d * 2, nb = (size_t)T * ((d + 31) / 32) * 4, ns = (size_t)T * 4;
+    if (overlap(X, nx, bits, nb) || overlap(X, nx, scale, ns) || overlap(bits, nb, scale, ns))
+        return SN_ERR_INVALID_ARG;
+    return cuda_status(sn::lossy_sign(X, T, d, bits, scale, (cudaStream_t)stream));
+}
+
+sn_status sn_sign_restore(const uint32_t *bits, const float *scale, int64_t T, int32_t d,
+                          void *X_out, sn_stream_t stream)
+{
+    sn_status st = check_batch(X_out, T, d);
+    if (st != SN_OK)
+        return st;
+    if (!bits || !scale)
+        return SN_ERR_INVALID_ARG;
+    if (!aligned(bits, 4) || !aligned(scale, 4))
+        return SN_ERR_ALIGNMENT;
+    if (T == 0)
+        return SN_OK;
+    const size_t nx = (size_t)T * d * 2;
+    if (overlap(X_out, nx, bits, (size_t)T * ((d + 31) / 32) * 4) ||
+        overlap(X_out, nx, scale, (size_t)T * 4))
+        return SN_ERR_INVALID_ARG;
+    return cuda_status(sn::lossy_sign_restore(bits, scale, T, d, X_out, (cudaStream_t)stream));
+}
+
 sn_status sn_wire_bytes(sn_basis_t b, sn_dtype dt, int64_t T, size_t *bytes)
 {
     if (!b || !bytes || T < 0 || (dt != SN_BF16 && dt != SN_F32))

@@ -88,6 +88,15 @@ cudaError_t grassmann_step(const sn_basis &b, const float *M, int K, float eta, 
 cudaError_t adamw_rowconst(bool grad_bf16, float *W, const void *g, float *M, float *V,
                            int64_t rows, int64_t cols, int64_t t, float lr, float b1, float b2,
                            float eps, float lam, float *colsum, cudaStream_t s);
+// Lossy comparators (bf16 batches [T, d])
+cudaError_t lossy_topk(const void *X, int64_t T, int d, int kk, void *vals, uint16_t *cols,
+                       cudaStream_t s);
+cudaError_t lossy_topk_restore(const void *vals, const uint16_t *cols, int64_t T, int d, int kk,
+                               void *out, cudaStream_t s);
+cudaError_t lossy_sign(const void *X, int64_t T, int d, uint32_t *bits, float *scale,
+                       cudaStream_t s);
+cudaError_t lossy_sign_restore(const uint32_t *bits, const float *scale, int64_t T, int d,
+                               void *out, cudaStream_t s);
 // C = X U - TU[ids] - PU[pos] (PU may be null)
 cudaError_t tc_compress_projected(const sn_basis &b, const __nv_bfloat16 *X, const int32_t *ids,
                                   const int32_t *pos, int64_t T, int seq_len, const float *TU,

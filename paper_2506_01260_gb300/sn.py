@@ -55,6 +55,10 @@ _sig("sn_grassmann_residual", [_P, _ST, _P, _P, _I64, _P, _P])
 _sig("sn_grassmann_step", [_P, _P, _I32, ctypes.c_float, _P, _P, _SZ, _P])
 _sig("sn_adamw_rowconst", [_ST, _P, _P, _P, _P, _I64, _I64, _I64, ctypes.c_float, ctypes.c_float,
                            ctypes.c_float, ctypes.c_float, ctypes.c_float, _P, _SZ, _P])
+_sig("sn_topk_compress", [_P, _I64, _I32, _I32, _P, _P, _P])
+_sig("sn_topk_restore", [_P, _P, _I64, _I32, _I32, _P, _P])
+_sig("sn_sign_compress", [_P, _I64, _I32, _P, _P, _P])
+_sig("sn_sign_restore", [_P, _P, _I64, _I32, _P, _P])
 _sig("sn_wire_bytes", [_P, _ST, _I64, ctypes.POINTER(_SZ)])
 _sig("sn_wire_send", [_P, _P, _SZ, _P])
 _sig("sn_wire_recv", [_P, _P, _SZ, _P])
@@ -68,7 +72,8 @@ EXPORTS = ["sn_basis_create", "sn_basis_destroy", "sn_basis_shape", "sn_compress
            "sn_project_weight_workspace", "sn_project_weight", "sn_project_weight_noalloc",
            "sn_project_tables", "sn_compress_fwd_projected", "sn_build_ts",
            "sn_grassmann_workspace", "sn_grassmann_accumulate", "sn_grassmann_residual",
-           "sn_grassmann_step", "sn_adamw_rowconst",
+           "sn_grassmann_step", "sn_adamw_rowconst", "sn_topk_compress", "sn_topk_restore",
+           "sn_sign_compress", "sn_sign_restore",
            "sn_wire_bytes", "sn_wire_send",
            "sn_wire_recv", "sn_check_errors", "sn_launch_count", "sn_status_string"]
 
@@ -318,6 +323,50 @@ def sn_adamw_rowconst(W, grad, M, V, step, lr, beta1=0.9, beta2=0.999, eps=1e-8,
                                   workspace.numel() * workspace.element_size(), _stream(stream)),
            "sn_adamw_rowconst")
     return W
+
+
+def sn_topk_compress(X, kk, stream=None):
+    """Per-row top-kk by magnitude of a bf16 batch: (values bf16 [T, kk], cols uint16-as-int16 [T, kk])."""
+    _need(X, "X", torch.bfloat16)
+    T, d = X.shape
+    vals = torch.empty(T, kk, dtype=torch.bfloat16, device=X.device)
+    cols = torch.empty(T, kk, dtype=torch.int16, device=X.device)
+    _check(_lib.sn_topk_compress(_ptr(X), T, d, kk, _ptr(vals), _ptr(cols), _stream(stream)),
+           "sn_topk_compress")
+    return vals, cols
+
+
+def sn_topk_restore(vals, cols, d, out=None, stream=None):
+    _need(vals, "values", torch.bfloat16)
+    _need(cols, "cols", torch.int16)
+    T, kk = vals.shape
+    if out is None:
+        out = torch.empty(T, d, dtype=torch.bfloat16, device=vals.device)
+    _check(_lib.sn_topk_restore(_ptr(vals), _ptr(cols), T, d, kk, _ptr(out), _stream(stream)),
+           "sn_topk_restore")
+    return out
+
+
+def sn_sign_compress(X, stream=None):
+    """1-bit signs (int32 words [T, ceil(d/32)]) and fp32 mean-magnitude row scales [T]."""
+    _need(X, "X", torch.bfloat16)
+    T, d = X.shape
+    bits = torch.empty(T, (d + 31) // 32, dtype=torch.int32, device=X.device)
+    scale = torch.empty(T, dtype=torch.float32, device=X.device)
+    _check(_lib.sn_sign_compress(_ptr(X), T, d, _ptr(bits), _ptr(scale), _stream(stream)),
+           "sn_sign_compress")
+    return bits, scale
+
+
+def sn_sign_restore(bits, scale, d, out=None, stream=None):
+    _need(bits, "bits", torch.int32)
+    _need(scale, "scale", torch.float32)
+    T = scale.shape[0]
+    if out is None:
+        out = torch.empty(T, d, dtype=torch.bfloat16, device=scale.device)
+    _check(_lib.sn_sign_restore(_ptr(bits), _ptr(scale), T, d, _ptr(out), _stream(stream)),
+           "sn_sign_restore")
+    return out
 
 
 def sn_decompress_fwd(basis, C, ids, tok_emb, seq_len, pos_emb=None, pos=None, out=None,
