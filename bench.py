@@ -285,6 +285,74 @@ def config_dict(workload=WORKLOAD):
                     "compute call; the receiving call waits on it"}
 
 
+# ---- lossy comparators at the codec's wire size ---------------------------------------
+
+def lossy_comparison(args, sn, basis, X, Xr, ids, tok, pe, n, flush, stream, hbm, pg, dev):
+    """Relative reconstruction error ||X' - X|| / ||X|| of the subspace codec and
+    of the lossy comparators on the same activation batch, with the wire bytes of
+    each: top-k at the codec's wire size (kk = k / 2: a bf16 value and a 16-bit
+    column per kept entry), sign quantization (1 bit per entry, the smallest
+    quantizer) and the randomized rank-r factorisation of the whole batch at the
+    codec's wire size (r = T k / (T + d)).  Top-k and sign are timed like the
+    step's kernels."""
+    import torch
+    from paper_2506_01260_gb300 import comparators
+
+    T, d = X.shape
+    k = basis.k
+    sn.sn_compress_fwd(basis, X, ids, tok, n, pos_emb=pe, out=torch.empty(T, k, dtype=X.dtype,
+                                                                           device=dev))
+    Xf = X.float()
+    xn = float(Xf.norm())
+
+    def rel(Xh):
+        return float((Xh.float() - Xf).norm()) / xn
+
+    def timed(fn, reps):
+        for _ in range(args.warmup):
+            flush.zero_()
+            fn()
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(reps)]
+        for a_, b_ in evs:
+            flush.zero_()
+            a_.record(stream)
+            fn()
+            b_.record(stream)
+        torch.cuda.synchronize()
+        return max_over_ranks(pg, statistics.mean(a_.elapsed_time(b_) for a_, b_ in evs), dev)
+
+    out = {"subspace": {"wire_bytes": 2 * T * k, "rel_error": rel(Xr)}}
+    kk = k // 2
+    vals = torch.empty(T, kk, dtype=X.dtype, device=dev)
+    cols = torch.empty(T, kk, dtype=torch.int16, device=dev)
+    tms = timed(lambda: sn.sn_topk_compress(X, kk, values=vals, cols=cols), min(args.steps, 20))
+    Xh, wb = comparators.topk_roundtrip(X, kk)
+    tab = 2 * T * d + 4 * T * kk
+    out["topk"] = {"kk": kk, "wire_bytes": wb, "rel_error": rel(Xh), "compress_ms": tms,
+                   "compress_gbs": tab / (tms / 1e3) / 1e9,
+                   "compress_frac": tab / (tms / 1e3) / 1e9 / hbm}
+    del Xh, vals, cols
+    words = (d + 31) // 32
+    bits = torch.empty(T, words, dtype=torch.int32, device=dev)
+    scale = torch.empty(T, dtype=torch.float32, device=dev)
+    sms = timed(lambda: sn.sn_sign_compress(X, bits=bits, scale=scale), min(args.steps, 20))
+    Xh, wb = comparators.sign_roundtrip(X)
+    sab = 2 * T * d + 4 * T * words + 4 * T
+    out["sign"] = {"wire_bytes": wb, "rel_error": rel(Xh), "compress_ms": sms,
+                   "compress_gbs": sab / (sms / 1e3) / 1e9,
+                   "compress_frac": sab / (sms / 1e3) / 1e9 / hbm}
+    del Xh, bits, scale
+    r = T * k // (T + d)
+    Xh, wb = comparators.lowrank_roundtrip(X, r)
+    out["lowrank"] = {"r": r, "wire_bytes": wb, "rel_error": rel(Xh)}
+    del Xh, Xf
+    out["note"] = ("same X as the step (embeddings + in-span signal + off-subspace noise); "
+                   "errors relative to ||X||; the codec subtracts the embeddings the "
+                   "receiver recomputes, the comparators send X itself")
+    return out
+
+
 # ---- our arm -------------------------------------------------------------------------
 
 def run_ours(args, world, rank, local, pg):
@@ -523,6 +591,8 @@ def run_ours(args, world, rank, local, pg):
             "note": "fp32 W, M, V, bf16 gradient; moments + column sums of V^ (pass 1), "
                     "W update with one rate per column (pass 2, re-reads M)"}
         del Wm, gW, Mm, Vm, aws
+        nxt["f4_lossy"] = lossy_comparison(args, sn, basis, X, Xr, ids, tok, pe, n, flush,
+                                           stream, hbm, pg, dev)
 
     # ---- end to end through the C ABI with host buffers ----
     e2e_line = None

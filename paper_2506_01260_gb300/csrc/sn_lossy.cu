@@ -1,105 +1,295 @@
 // sn_lossy.cu — the lossy comparators of the paper's comparison at equal wire
 // size (Sec. 8, "Comparison against lossy compressions"): per-row top-k and
-// 1-bit sign quantization of a bf16 batch, with their restores.  One CTA per
-// row (grid-stride over rows), 256 threads.
+// 1-bit sign quantization of a bf16 batch, with their restores.
 //
 // Top-k keeps the kk entries of largest magnitude of each row, ties towards the
-// lower column, and writes them in ascending column order.  The threshold
-// magnitude is found exactly by a two-pass radix select on the 15-bit bf16
-// magnitude (high 8 bits, then low 7); a third pass scans the row in column
-// order (warp ballots) to place the kept entries and to take, among entries
-// equal to the threshold, the lowest columns first.
-#include "sn_internal.cuh"
+// lower column, and writes them in ascending column order.  One warp per row
+// (grid-stride over rows, 8 warps a CTA, no block barriers); selection works
+// on the 15-bit bf16 magnitude ("key"), lane l owning chunks l, l + 32, ... of
+// 8 entries (16 bytes).
+//
+//   bound   Lane l keeps the M largest maxima of its chunks; the bound is the
+//           q-th largest, over the lanes, of each lane's M-th (q = ceil(kk/M)).
+//           q lanes then vouch for M distinct chunks each whose maximum
+//           reaches the bound, so at least kk entries do: the kk-th largest
+//           key is >= bound.  M = ceil(kk / 24), at most 4.
+//   select  The chunks whose maximum reaches the bound are re-read (they are
+//           still in L2) and their entries at or above it appended in column
+//           order (about 2 kk of them on continuous data); the kk-th largest
+//           key among those is found by a bit-by-bit search with warp counts,
+//           and the kept entries are placed by ballot prefixes, the lowest
+//           columns first among those equal to it.
+//   exact   When more than kWCap chunks or entries reach the bound (many
+//           equal keys, kk > 128) the same search and placement run over the
+//           whole row, re-read from L2, skipping chunks whose maximum cannot
+//           matter.
+#include "sn_tc.cuh"
 
 namespace sn {
 namespace {
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
+constexpr int kWCap = 256;                // candidate chunks and entries per warp
+constexpr int kLoadBatch = 8;             // 16-byte loads in flight per lane (top-k)
+constexpr int kSignUnroll = 8;            // 16-byte loads in flight per lane (sign)
 
-// Exclusive prefix of `flag` over the block in thread order and the block
-// total; all threads must call it.  `ws` holds kWarps ints of shared memory.
-__device__ __forceinline__ int block_scan(bool flag, int *ws, int &total)
+__device__ __forceinline__ uint32_t max_u16x2(uint32_t a, uint32_t b)
 {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const unsigned m = __ballot_sync(0xffffffffu, flag);
-    __syncthreads();                          // ws free from the previous scan
-    if (lane == 0)
-        ws[warp] = __popc(m);
-    __syncthreads();
-    int before = 0;
-    total = 0;
-    for (int w = 0; w < kWarps; ++w) {
-        before += w < warp ? ws[w] : 0;
-        total += ws[w];
-    }
-    return before + __popc(m & ((1u << lane) - 1u));
+    uint32_t r;
+    asm("max.u16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+    return r;
 }
 
+// Largest magnitude key among the 8 bf16 of a chunk.
+__device__ __forceinline__ int max_key8(uint4 v)
+{
+    const uint32_t c = max_u16x2(max_u16x2(v.x & 0x7FFF7FFFu, v.y & 0x7FFF7FFFu),
+                                 max_u16x2(v.z & 0x7FFF7FFFu, v.w & 0x7FFF7FFFu));
+    return (int)max(c & 0xFFFFu, c >> 16);
+}
+
+__device__ __forceinline__ int key_of(uint4 v, int e)
+{
+    const uint32_t w = e < 2 ? v.x : e < 4 ? v.y : e < 6 ? v.z : v.w;
+    return (int)((w >> (16 * (e & 1))) & 0x7FFFu);
+}
+
+__device__ __forceinline__ uint32_t bits_of(uint4 v, int e)
+{
+    const uint32_t w = e < 2 ? v.x : e < 4 ? v.y : e < 6 ? v.z : v.w;
+    return (w >> (16 * (e & 1))) & 0xFFFFu;
+}
+
+__device__ __forceinline__ int warp_count(bool p) { return __popc(__ballot_sync(0xffffffffu, p)); }
+
+__device__ __forceinline__ uint32_t lanes_below()
+{
+    return (1u << (threadIdx.x & 31)) - 1u;
+}
+
+// Inclusive prefix sum over the warp.
+__device__ __forceinline__ int warp_incl_scan(int n)
+{
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, n, o);
+        n += lane >= o ? y : 0;
+    }
+    return n;
+}
+
+// Count of the chunk's entries whose key is >= thr.
+__device__ __forceinline__ int count_ge8(uint4 v, int thr)
+{
+    int n = 0;
+#pragma unroll
+    for (int e = 0; e < 8; ++e)
+        n += key_of(v, e) >= thr;
+    return n;
+}
+
+// Shared memory of one warp: chunk maxima, candidate chunks, candidate
+// entries (bf16 bits | column << 16).
+struct TopkWarpSmem {
+    uint16_t *smax;
+    uint16_t *clist;
+    uint32_t *cand;
+};
+
+__host__ __device__ __forceinline__ int topk_region_bytes(int nch)
+{
+    return ((nch * 2 + 15) & ~15) + kWCap * 2 + kWCap * 4;
+}
+
+// Exact path: the kk-th largest key of the whole row and the placement of
+// the kept entries in column order.
+__device__ void topk_row_exact(const uint4 *src, int nch, int kk, const uint16_t *smax,
+                               uint16_t *vo, uint16_t *co)
+{
+    const int lane = threadIdx.x & 31;
+    int thr = 0;
+    for (int bit = 14; bit >= 0; --bit) {
+        const int trial = thr | (1 << bit);
+        int cnt = 0;
+        for (int c = lane; c < nch; c += 32)
+            if ((int)smax[c] >= trial)
+                cnt += count_ge8(__ldg(src + c), trial);
+        if (__reduce_add_sync(0xffffffffu, cnt) >= kk)
+            thr = trial;
+    }
+    int above = 0;
+    for (int c = lane; c < nch; c += 32)
+        if ((int)smax[c] > thr)
+            above += count_ge8(__ldg(src + c), thr + 1);
+    const int need = kk - __reduce_add_sync(0xffffffffu, above);
+    int eq_before = 0, kept_before = 0;
+    for (int c0 = 0; c0 < nch; c0 += 32) {                    // warp-uniform
+        const int c = c0 + lane;
+        const bool live = c < nch && (int)smax[c] >= thr;
+        const uint4 v = live ? __ldg(src + c) : make_uint4(0, 0, 0, 0);
+        uint32_t eqf = 0, gtf = 0;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const int k = live ? key_of(v, e) : -1;
+            eqf |= (k == thr ? 1u : 0u) << e;
+            gtf |= (k > thr ? 1u : 0u) << e;
+        }
+        const int neq = __popc(eqf);
+        const int eq_incl = warp_incl_scan(neq);
+        int allowed = need - (eq_before + eq_incl - neq);     // ties this lane may still take
+        uint32_t keep = gtf, rest = eqf;
+        while (allowed > 0 && rest) {
+            const uint32_t low = rest & (0u - rest);
+            keep |= low;
+            rest ^= low;
+            --allowed;
+        }
+        const int nk = __popc(keep);
+        const int k_incl = warp_incl_scan(nk);
+        int p = kept_before + k_incl - nk;
+#pragma unroll
+        for (int e = 0; e < 8; ++e)
+            if ((keep >> e) & 1u) {
+                vo[p] = (uint16_t)bits_of(v, e);
+                co[p] = (uint16_t)(8 * c + e);
+                ++p;
+            }
+        eq_before += __shfl_sync(0xffffffffu, eq_incl, 31);
+        kept_before += __shfl_sync(0xffffffffu, k_incl, 31);
+    }
+}
+
+template <int M>
 __global__ void __launch_bounds__(kThreads) k_topk(const uint16_t *__restrict__ X, int64_t T,
                                                     int d, int kk, uint16_t *__restrict__ vals,
                                                     uint16_t *__restrict__ cols)
 {
-    extern __shared__ uint16_t row[];         // d bf16 patterns
-    __shared__ int hist[256];
-    __shared__ int ws[kWarps];
-    __shared__ int sel[4];                    // bin, threshold, above, need
-    for (int64_t t = blockIdx.x; t < T; t += gridDim.x) {
-        const uint16_t *src = X + t * (int64_t)d;
-        __syncthreads();
-        for (int c = threadIdx.x; c < d / 8; c += kThreads)
-            ((uint4 *)row)[c] = __ldg((const uint4 *)src + c);
-        for (int c = threadIdx.x; c < 256; c += kThreads)
-            hist[c] = 0;
-        __syncthreads();
-        // pass 1: high 8 bits of the magnitude
-        for (int c = threadIdx.x; c < d; c += kThreads)
-            atomicAdd(&hist[(row[c] & 0x7FFF) >> 7], 1);
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            int above = 0, b = 255;
-            while (above + hist[b] < kk)
-                above += hist[b--];
-            sel[0] = b;
-            sel[2] = above;
-        }
-        __syncthreads();
-        const int B = sel[0];
-        for (int c = threadIdx.x; c < 128; c += kThreads)
-            hist[c] = 0;
-        __syncthreads();
-        // pass 2: low 7 bits of the entries in bin B
-        for (int c = threadIdx.x; c < d; c += kThreads) {
-            const int m = row[c] & 0x7FFF;
-            if ((m >> 7) == B)
-                atomicAdd(&hist[m & 127], 1);
-        }
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            int above = sel[2], l = 127;
-            while (above + hist[l] < kk)
-                above += hist[l--];
-            sel[1] = (B << 7) | l;
-            sel[2] = above;
-            sel[3] = kk - above;
-        }
-        __syncthreads();
-        const int thr = sel[1], need = sel[3];
-        // pass 3: place the kept entries in column order
-        int kept = 0, eqs = 0;
-        for (int c0 = 0; c0 < d; c0 += kThreads) {
-            const int c = c0 + threadIdx.x;
-            const int m = c < d ? (row[c] & 0x7FFF) : -1;
-            int eq_total, keep_total;
-            const int eq_rank = eqs + block_scan(m == thr, ws, eq_total);
-            const bool keep = m > thr || (m == thr && eq_rank < need);
-            const int slot = kept + block_scan(keep, ws, keep_total);
-            if (keep) {
-                vals[t * kk + slot] = row[c];
-                cols[t * kk + slot] = (uint16_t)c;
+    extern __shared__ __align__(16) uint8_t tk_smem[];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int nch = d / 8, per_lane = (nch + 31) / 32;
+    uint8_t *base = tk_smem + warp * topk_region_bytes(nch);
+    uint16_t *smax = (uint16_t *)base;
+    uint16_t *clist = (uint16_t *)(base + ((nch * 2 + 15) & ~15));
+    uint32_t *cand = (uint32_t *)(base + ((nch * 2 + 15) & ~15) + kWCap * 2);
+    const int q = M > 0 ? (kk + M - 1) / M : 33;
+    const int64_t nwarps = (int64_t)gridDim.x * kWarps;
+    for (int64_t t = (int64_t)blockIdx.x * kWarps + warp; t < T; t += nwarps) {
+        const uint4 *src = (const uint4 *)(X + t * (int64_t)d);
+        uint16_t *vo = vals + t * kk;
+        uint16_t *co = cols + t * kk;
+        __syncwarp();                         // the previous row is done with smax, clist, cand
+        // pass 1: chunk maxima, and each lane's M largest
+        int top[M > 0 ? M : 1];
+#pragma unroll
+        for (int j = 0; j < (M > 0 ? M : 1); ++j)
+            top[j] = -1;
+        for (int i0 = 0; i0 < per_lane; i0 += kLoadBatch) {
+            uint4 v[kLoadBatch];
+#pragma unroll
+            for (int u = 0; u < kLoadBatch; ++u) {
+                const int c = lane + 32 * (i0 + u);
+                v[u] = c < nch ? __ldg(src + c) : make_uint4(0, 0, 0, 0);
             }
-            kept += keep_total;
-            eqs += eq_total;
+#pragma unroll
+            for (int u = 0; u < kLoadBatch; ++u) {
+                const int c = lane + 32 * (i0 + u);
+                if (c < nch) {
+                    int x = max_key8(v[u]);
+                    smax[c] = (uint16_t)x;
+#pragma unroll
+                    for (int j = 0; j < M; ++j) {
+                        const int hi = max(top[j], x);
+                        x = min(top[j], x);
+                        top[j] = hi;
+                    }
+                }
+            }
+        }
+        int bound = -1;
+        if (M > 0 && q <= 32) {
+            const int vl = top[M > 0 ? M - 1 : 0];
+            int b = 0;
+            for (int bit = 14; bit >= 0; --bit)
+                if (warp_count(vl >= (b | (1 << bit))) >= q)
+                    b |= 1 << bit;
+            bound = warp_count(vl >= b) >= q ? b : -1;
+        }
+        __syncwarp();                         // smax visible to the whole warp
+        // candidate chunks, in column order
+        int nchk = 0;
+        for (int i = 0; i < per_lane; ++i) {
+            const int c = lane + 32 * i;
+            const bool hit = c < nch && (int)smax[c] >= bound;
+            const uint32_t bal = __ballot_sync(0xffffffffu, hit);
+            const int p = nchk + __popc(bal & lanes_below());
+            if (hit && p < kWCap)
+                clist[p] = (uint16_t)c;
+            nchk += __popc(bal);
+        }
+        bool exact = nchk > kWCap;
+        int nc = 0;
+        if (!exact) {
+            __syncwarp();
+            for (int r0 = 0; r0 < nchk; r0 += 32) {           // warp-uniform
+                const int j = r0 + lane;
+                const int c = j < nchk ? (int)clist[j] : 0;
+                const uint4 v = j < nchk ? __ldg(src + c) : make_uint4(0, 0, 0, 0);
+                uint32_t f = 0;
+#pragma unroll
+                for (int e = 0; e < 8; ++e)
+                    f |= (j < nchk && key_of(v, e) >= bound ? 1u : 0u) << e;
+                const int n = __popc(f);
+                const int incl = warp_incl_scan(n);
+                int p = nc + incl - n;
+#pragma unroll
+                for (int e = 0; e < 8; ++e)
+                    if ((f >> e) & 1u) {
+                        if (p < kWCap)
+                            cand[p] = bits_of(v, e) | ((uint32_t)(8 * c + e) << 16);
+                        ++p;
+                    }
+                nc += __shfl_sync(0xffffffffu, incl, 31);
+            }
+            exact = nc > kWCap;
+        }
+        if (exact) {
+            topk_row_exact(src, nch, kk, smax, vo, co);
+            continue;
+        }
+        __syncwarp();                         // cand visible to the whole warp
+        // every entry at or above the bound is a candidate, so for any trial
+        // the candidate count decides "at least kk entries reach it" as the
+        // whole row would
+        int thr = 0;
+        for (int bit = 14; bit >= 0; --bit) {
+            const int trial = thr | (1 << bit);
+            int cnt = 0;
+            for (int j = lane; j < nc; j += 32)
+                cnt += (int)(cand[j] & 0x7FFFu) >= trial;
+            if (__reduce_add_sync(0xffffffffu, cnt) >= kk)
+                thr = trial;
+        }
+        int above = 0;
+        for (int j = lane; j < nc; j += 32)
+            above += (int)(cand[j] & 0x7FFFu) > thr;
+        const int need = kk - __reduce_add_sync(0xffffffffu, above);
+        int eq_before = 0, kept_before = 0;
+        for (int r0 = 0; r0 < nc; r0 += 32) {                 // warp-uniform
+            const int j = r0 + lane;
+            const uint32_t cj = j < nc ? cand[j] : 0u;
+            const int k = j < nc ? (int)(cj & 0x7FFFu) : -1;
+            const uint32_t be = __ballot_sync(0xffffffffu, k == thr);
+            const bool keep = k > thr || (k == thr && eq_before + __popc(be & lanes_below()) < need);
+            const uint32_t bk = __ballot_sync(0xffffffffu, keep);
+            if (keep) {
+                const int p = kept_before + __popc(bk & lanes_below());
+                vo[p] = (uint16_t)(cj & 0xFFFFu);
+                co[p] = (uint16_t)(cj >> 16);
+            }
+            eq_before += __popc(be);
+            kept_before += __popc(bk);
         }
     }
 }
@@ -120,50 +310,83 @@ __global__ void __launch_bounds__(kThreads) k_topk_restore(const uint16_t *__res
     }
 }
 
+// Sign quantization: one warp per row; lane l of a 256-column slab reads its
+// 8 entries as one 16-byte load, forms their 8 sign bits (1 for a negative
+// nonzero entry; NaN inputs are outside the comparator's domain), and 4 lanes
+// merge their bytes into one 32-bit word.  The row scale is the mean
+// magnitude, summed per chunk, then per lane, then across the warp in fp32.
 __global__ void __launch_bounds__(kThreads) k_sign(const uint16_t *__restrict__ X, int64_t T, int d,
                                                     uint32_t *__restrict__ bits,
                                                     float *__restrict__ scale)
 {
-    __shared__ float red[kWarps];
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int words = (d + 31) / 32;
-    for (int64_t t = blockIdx.x; t < T; t += gridDim.x) {
-        const uint16_t *src = X + t * (int64_t)d;
+    const int lane = threadIdx.x & 31;
+    const int64_t nwarps = ((int64_t)gridDim.x * kThreads) >> 5;
+    const int nch = d / 8, words = (d + 31) / 32;
+    for (int64_t t = ((int64_t)blockIdx.x * kThreads + threadIdx.x) >> 5; t < T; t += nwarps) {
+        const uint4 *src = (const uint4 *)(X + t * (int64_t)d);
+        uint32_t *dst = bits + t * words;
         float s = 0.f;
-        for (int w = warp; w < words; w += kWarps) {
-            const int c = 32 * w + lane;
-            const uint16_t b = c < d ? src[c] : (uint16_t)0;
-            s += __uint_as_float((uint32_t)(b & 0x7FFF) << 16);
-            const unsigned m = __ballot_sync(0xffffffffu, (b & 0x8000) && (b & 0x7FFF));
-            if (lane == 0)
-                bits[t * words + w] = m;
+        for (int base = 0; base < nch; base += kSignUnroll * 32) {     // warp-uniform
+            uint4 v[kSignUnroll];
+#pragma unroll
+            for (int u = 0; u < kSignUnroll; ++u) {
+                const int c = base + 32 * u + lane;
+                v[u] = c < nch ? __ldg(src + c) : make_uint4(0, 0, 0, 0);
+            }
+#pragma unroll
+            for (int u = 0; u < kSignUnroll; ++u) {
+                const int c = base + 32 * u + lane;
+                const uint32_t wd[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+                // per 32-bit word: sign AND "magnitude nonzero" (adding 0x7FFF
+                // to a 15-bit magnitude carries into bit 15 exactly when it is
+                // not 0), moved so word e's two bits land on 2e and 16 + 2e
+                uint32_t x = 0;
+                float cs = 0.f;
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const uint32_t w = wd[e];
+                    x |= (w & ((w & 0x7FFF7FFFu) + 0x7FFF7FFFu) & 0x80008000u) >> (15 - 2 * e);
+                    cs += fabsf(__uint_as_float(w << 16)) + fabsf(__uint_as_float(w & 0xFFFF0000u));
+                }
+                const uint32_t byte = (x | (x >> 15)) & 0xFFu;
+                s += cs;
+                uint32_t wv = byte << (8 * (lane & 3));
+                wv |= __shfl_xor_sync(0xffffffffu, wv, 1);
+                wv |= __shfl_xor_sync(0xffffffffu, wv, 2);
+                if ((lane & 3) == 0 && (c >> 2) < words)
+                    dst[c >> 2] = wv;
+            }
         }
+#pragma unroll
         for (int o = 16; o > 0; o >>= 1)
             s += __shfl_xor_sync(0xffffffffu, s, o);
-        __syncthreads();
         if (lane == 0)
-            red[warp] = s;
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            float tot = 0.f;
-            for (int w = 0; w < kWarps; ++w)
-                tot += red[w];
-            scale[t] = tot / (float)d;
-        }
+            scale[t] = s / (float)d;
     }
 }
 
-__global__ void k_sign_restore(const uint32_t *__restrict__ bits, const float *__restrict__ scale,
-                               int64_t T, int d, __nv_bfloat16 *__restrict__ out)
+// Restore: one warp per row, one 16-byte store of 8 entries per lane.
+__global__ void __launch_bounds__(kThreads) k_sign_restore(const uint32_t *__restrict__ bits,
+                                                            const float *__restrict__ scale,
+                                                            int64_t T, int d,
+                                                            uint16_t *__restrict__ out)
 {
-    const int words = (d + 31) / 32;
-    const int64_t n = T * (int64_t)d;
-    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n;
-         e += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t t = e / d;
-        const int c = (int)(e - t * d);
-        const bool neg = (bits[t * words + c / 32] >> (c & 31)) & 1u;
-        out[e] = __float2bfloat16_rn(neg ? -scale[t] : scale[t]);
+    const int lane = threadIdx.x & 31;
+    const int64_t nwarps = ((int64_t)gridDim.x * kThreads) >> 5;
+    const int nch = d / 8, words = (d + 31) / 32;
+    for (int64_t t = ((int64_t)blockIdx.x * kThreads + threadIdx.x) >> 5; t < T; t += nwarps) {
+        const __nv_bfloat16 pos = __float2bfloat16_rn(scale[t]);
+        const __nv_bfloat16 neg = __float2bfloat16_rn(-scale[t]);
+        const uint32_t p = *(const uint16_t *)&pos, n = *(const uint16_t *)&neg;
+        uint4 *dst = (uint4 *)(out + t * (int64_t)d);
+        for (int c = lane; c < nch; c += 32) {
+            const uint32_t byte = (bits[t * words + (c >> 2)] >> (8 * (c & 3))) & 0xFFu;
+            uint32_t wd[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+                wd[e] = ((byte >> (2 * e)) & 1u ? n : p) | (((byte >> (2 * e + 1)) & 1u ? n : p) << 16);
+            dst[c] = make_uint4(wd[0], wd[1], wd[2], wd[3]);
+        }
     }
 }
 
@@ -175,20 +398,54 @@ int row_grid(int64_t T)
     return (int)(T < 8 * (int64_t)sms ? T : 8 * (int64_t)sms);
 }
 
+// One warp per row: at most 8 resident CTAs of 8 warps per SM.
+int warp_grid(int64_t T)
+{
+    int dev = 0, sms = 148;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int64_t need = (T + kWarps - 1) / kWarps;
+    return (int)(need < 8 * (int64_t)sms ? need : 8 * (int64_t)sms);
+}
+
+template <int M>
+cudaError_t launch_topk(const void *X, int64_t T, int d, int kk, void *vals, uint16_t *cols,
+                        cudaStream_t s)
+{
+    const size_t smem = (size_t)kWarps * topk_region_bytes(d / 8);
+    cudaError_t e = cudaFuncSetAttribute(k_topk<M>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess)
+        return e;
+    int dev = 0, sms = 148, per_sm = 1;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_topk<M>, kThreads, smem);
+    if (e != cudaSuccess)
+        return e;
+    const int64_t resident = (int64_t)sms * (per_sm > 0 ? per_sm : 1);   // one wave
+    const int64_t need = (T + kWarps - 1) / kWarps;
+    k_topk<M><<<(int)(need < resident ? need : resident), kThreads, smem, s>>>(
+        (const uint16_t *)X, T, d, kk, (uint16_t *)vals, cols);
+    count_launch();
+    return cudaGetLastError();
+}
+
 }  // namespace
 
 cudaError_t lossy_topk(const void *X, int64_t T, int d, int kk, void *vals, uint16_t *cols,
                        cudaStream_t s)
 {
-    const size_t smem = sizeof(uint16_t) * (size_t)d;
-    cudaError_t e = cudaFuncSetAttribute(k_topk, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
-    if (e != cudaSuccess)
-        return e;
-    k_topk<<<row_grid(T), kThreads, smem, s>>>((const uint16_t *)X, T, d, kk, (uint16_t *)vals,
-                                                cols);
-    count_launch();
-    return cudaGetLastError();
+    // M = ceil(kk / 24) chunk maxima vouched for per lane; past 4 the bound
+    // is too loose to pay and every row takes the exact path
+    const int m = (kk + 23) / 24;
+    switch (m) {
+    case 1: return launch_topk<1>(X, T, d, kk, vals, cols, s);
+    case 2: return launch_topk<2>(X, T, d, kk, vals, cols, s);
+    case 3: return launch_topk<3>(X, T, d, kk, vals, cols, s);
+    case 4: return launch_topk<4>(X, T, d, kk, vals, cols, s);
+    default: return launch_topk<0>(X, T, d, kk, vals, cols, s);
+    }
 }
 
 cudaError_t lossy_topk_restore(const void *vals, const uint16_t *cols, int64_t T, int d, int kk,
@@ -203,7 +460,7 @@ cudaError_t lossy_topk_restore(const void *vals, const uint16_t *cols, int64_t T
 cudaError_t lossy_sign(const void *X, int64_t T, int d, uint32_t *bits, float *scale,
                        cudaStream_t s)
 {
-    k_sign<<<row_grid(T), kThreads, 0, s>>>((const uint16_t *)X, T, d, bits, scale);
+    k_sign<<<warp_grid(T), kThreads, 0, s>>>((const uint16_t *)X, T, d, bits, scale);
     count_launch();
     return cudaGetLastError();
 }
@@ -211,7 +468,7 @@ cudaError_t lossy_sign(const void *X, int64_t T, int d, uint32_t *bits, float *s
 cudaError_t lossy_sign_restore(const uint32_t *bits, const float *scale, int64_t T, int d,
                                void *out, cudaStream_t s)
 {
-    k_sign_restore<<<4 * row_grid(T), 256, 0, s>>>(bits, scale, T, d, (__nv_bfloat16 *)out);
+    k_sign_restore<<<warp_grid(T), kThreads, 0, s>>>(bits, scale, T, d, (uint16_t *)out);
     count_launch();
     return cudaGetLastError();
 }

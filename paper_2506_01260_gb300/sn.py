@@ -325,12 +325,18 @@ def sn_adamw_rowconst(W, grad, M, V, step, lr, beta1=0.9, beta2=0.999, eps=1e-8,
     return W
 
 
-def sn_topk_compress(X, kk, stream=None):
+def sn_topk_compress(X, kk, values=None, cols=None, stream=None):
     """Per-row top-kk by magnitude of a bf16 batch: (values bf16 [T, kk], cols uint16-as-int16 [T, kk])."""
     _need(X, "X", torch.bfloat16)
     T, d = X.shape
-    vals = torch.empty(T, kk, dtype=torch.bfloat16, device=X.device)
-    cols = torch.empty(T, kk, dtype=torch.int16, device=X.device)
+    vals = values if values is not None else torch.empty(T, kk, dtype=torch.bfloat16,
+                                                         device=X.device)
+    if cols is None:
+        cols = torch.empty(T, kk, dtype=torch.int16, device=X.device)
+    _need(vals, "values", torch.bfloat16)
+    _need(cols, "cols", torch.int16)
+    if vals.shape != (T, kk) or cols.shape != (T, kk):
+        raise ValueError("values and cols must be [T, kk]")
     _check(_lib.sn_topk_compress(_ptr(X), T, d, kk, _ptr(vals), _ptr(cols), _stream(stream)),
            "sn_topk_compress")
     return vals, cols
@@ -347,12 +353,18 @@ def sn_topk_restore(vals, cols, d, out=None, stream=None):
     return out
 
 
-def sn_sign_compress(X, stream=None):
+def sn_sign_compress(X, bits=None, scale=None, stream=None):
     """1-bit signs (int32 words [T, ceil(d/32)]) and fp32 mean-magnitude row scales [T]."""
     _need(X, "X", torch.bfloat16)
     T, d = X.shape
-    bits = torch.empty(T, (d + 31) // 32, dtype=torch.int32, device=X.device)
-    scale = torch.empty(T, dtype=torch.float32, device=X.device)
+    if bits is None:
+        bits = torch.empty(T, (d + 31) // 32, dtype=torch.int32, device=X.device)
+    if scale is None:
+        scale = torch.empty(T, dtype=torch.float32, device=X.device)
+    _need(bits, "bits", torch.int32)
+    _need(scale, "scale", torch.float32)
+    if bits.shape != (T, (d + 31) // 32) or scale.shape != (T,):
+        raise ValueError("bits must be [T, ceil(d/32)] and scale [T]")
     _check(_lib.sn_sign_compress(_ptr(X), T, d, _ptr(bits), _ptr(scale), _stream(stream)),
            "sn_sign_compress")
     return bits, scale

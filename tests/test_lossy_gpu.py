@@ -26,19 +26,28 @@ def lossy_oracle():
     return mod
 
 
-def batch(T, d, seed, ties=False):
+def batch(T, d, seed, ties=False, const=False):
     rng = np.random.default_rng(seed)
     x = rng.standard_normal((T, d))
     if ties:                                           # many equal magnitudes
         x = np.round(x * 2) / 2
+    if const:                                          # one magnitude per row, random signs
+        x = np.sign(x) * rng.uniform(0.5, 2.0, (T, 1))
     return W.to_bf16(x)
 
 
-@pytest.mark.parametrize("T,d,kk,ties", [(300, 512, 41, False), (20, 8192, 41, False),
-                                          (64, 256, 30, True), (9, 64, 64, True), (5, 128, 1, False)])
-def test_topk_bit_exact(sn, T, d, kk, ties):
+# Most cases take the candidate path (few entries reach the bound, M = 1..4
+# chunk maxima vouched for per lane); kk > 96, rows of one magnitude and
+# heavy ties on wide rows take the exact whole-row path.
+@pytest.mark.parametrize("T,d,kk,ties,const", [
+    (300, 512, 41, False, False), (20, 8192, 41, False, False), (64, 256, 30, True, False),
+    (9, 64, 64, True, False), (5, 128, 1, False, False), (40, 2048, 256, True, False),
+    (4, 8192, 300, False, False), (3, 4096, 41, False, True), (6, 256, 17, False, True),
+    (2, 65536, 4096, False, False), (50, 4096, 70, False, False), (50, 4096, 90, False, False),
+    (33, 8200, 41, False, False)])
+def test_topk_bit_exact(sn, T, d, kk, ties, const):
     o = lossy_oracle()
-    xb = batch(T, d, seed=T + d, ties=ties)
+    xb = batch(T, d, seed=T + d, ties=ties, const=const)
     vals, cols = sn.sn_topk_compress(dev(xb), kk)
     c = host(cols).view(np.uint16).astype(np.int64)
     ref_cols = o.topk_columns(xb, kk)
