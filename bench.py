@@ -80,10 +80,12 @@ def algorithmic_bytes(T, d, k, n, u, m_cols, s=2):
 
 
 def kernel_sources_sha1():
+    """Hash of the sources the step's kernels and their launch set-up are
+    built from (the tensor-core kernels, their host side and headers)."""
     import glob
     import hashlib
     h = hashlib.sha1()
-    for p in sorted(glob.glob(os.path.join(ROOT, "paper_2506_01260_gb300", "csrc", "*.cu*"))):
+    for p in sorted(glob.glob(os.path.join(ROOT, "paper_2506_01260_gb300", "csrc", "sn_tc*.cu*"))):
         h.update(os.path.basename(p).encode())
         with open(p, "rb") as f:
             h.update(f.read())
