@@ -610,34 +610,48 @@ def run_ours(args, world, rank, local, pg):
         h2d = Xh.numel() * 2 + Gh.numel() * 2 + idsh.numel() * 4
         d2h = Xoh.numel() * 2 + Goh.numel() * 2
 
-        # Host copies ride their own streams: G's upload overlaps the forward
-        # compress, X' downloads while the gradient recover runs, and one step's
-        # downloads overlap the next step's uploads (the link runs both
-        # directions at once).  Every step still copies its own inputs in and
-        # its results out; events keep each buffer from being overwritten while
-        # it is read or sent.
+        # Host copies ride their own streams and the device side of every host
+        # buffer is doubled, so the link never waits for compute: step i + 1's
+        # uploads start as soon as step i's are done (X, ids and G of the step
+        # before last have been read by then), and each step's X' and G' leave
+        # while the next step's inputs arrive (the link runs both directions at
+        # once).  Every step still copies its own inputs in and its results
+        # out; events keep each buffer from being overwritten while it is read
+        # or sent.
         h2d_stream = torch.cuda.Stream()
         d2h_stream = torch.cuda.Stream()
-        cev = [torch.cuda.Event() for _ in range(6)]
-        for e_ in cev[4:]:
-            e_.record(d2h_stream)
+        Xd, Gd, idsd = [X, torch.empty_like(X)], [G, torch.empty_like(G)], [ids, torch.empty_like(ids)]
+        Xrd, Grd = [Xr, torch.empty_like(Xr)], [Gr, torch.empty_like(Gr)]
+        ev = {name: [torch.cuda.Event() for _ in range(2)]
+              for name in ("x_free", "g_free", "x_in", "g_in", "xr_done", "gr_done", "xr_free",
+                           "gr_free")}
+        for b_ in range(2):
+            for name in ("x_free", "g_free"):
+                ev[name][b_].record(stream)
+            for name in ("xr_free", "gr_free"):
+                ev[name][b_].record(d2h_stream)
+        step_no = [0]
 
         def e2e_step():
-            h2d_stream.wait_stream(stream)          # the previous step is done with X, G
-            sn.sn_wire_recv(Xh, X, stream=h2d_stream)
-            sn.sn_wire_recv(idsh, ids, stream=h2d_stream)
-            cev[0].record(h2d_stream)
-            sn.sn_wire_recv(Gh, G, stream=h2d_stream)
-            cev[1].record(h2d_stream)
-            stream.wait_event(cev[0])
-            sn.sn_compress_fwd(basis, X, ids, tok, n, pos_emb=pe, out=C)
+            b_ = step_no[0] % 2
+            step_no[0] += 1
+            h2d_stream.wait_event(ev["x_free"][b_])     # X, ids of two steps ago are read
+            sn.sn_wire_recv(Xh, Xd[b_], stream=h2d_stream)
+            sn.sn_wire_recv(idsh, idsd[b_], stream=h2d_stream)
+            ev["x_in"][b_].record(h2d_stream)
+            h2d_stream.wait_event(ev["g_free"][b_])
+            sn.sn_wire_recv(Gh, Gd[b_], stream=h2d_stream)
+            ev["g_in"][b_].record(h2d_stream)
+            stream.wait_event(ev["x_in"][b_])
+            sn.sn_compress_fwd(basis, Xd[b_], idsd[b_], tok, n, pos_emb=pe, out=C)
             sync_ev[0].record(stream)
             wire_stream.wait_event(sync_ev[0])
             sn.sn_wire_send(C, wire_f, stream=wire_stream)
             sn.sn_wire_recv(wire_f, C_rx, stream=wire_stream)
             sync_ev[1].record(wire_stream)
-            stream.wait_event(cev[1])
-            sn.sn_compress_bwd(basis, G, out=Cg)
+            stream.wait_event(ev["g_in"][b_])
+            sn.sn_compress_bwd(basis, Gd[b_], out=Cg)
+            ev["g_free"][b_].record(stream)
             sync_ev[2].record(stream)
             wire_stream.wait_event(sync_ev[2])
             sn.sn_wire_send(Cg, wire_b, stream=wire_stream)
@@ -645,19 +659,20 @@ def run_ours(args, world, rank, local, pg):
             sync_ev[3].record(wire_stream)
             sn.sn_project_weight(basis, Wo, out=Wp, workspace=ws)
             stream.wait_event(sync_ev[1])
-            stream.wait_event(cev[4])               # the previous X' has left
-            sn.sn_decompress_fwd(basis, C_rx, ids, tok, n, pos_emb=pe, out=Xr)
-            cev[2].record(stream)
-            d2h_stream.wait_event(cev[2])
-            sn.sn_wire_send(Xr, Xoh, stream=d2h_stream)
-            cev[4].record(d2h_stream)
+            stream.wait_event(ev["xr_free"][b_])         # X' of two steps ago has left
+            sn.sn_decompress_fwd(basis, C_rx, idsd[b_], tok, n, pos_emb=pe, out=Xrd[b_])
+            ev["x_free"][b_].record(stream)
+            ev["xr_done"][b_].record(stream)
+            d2h_stream.wait_event(ev["xr_done"][b_])
+            sn.sn_wire_send(Xrd[b_], Xoh, stream=d2h_stream)
+            ev["xr_free"][b_].record(d2h_stream)
             stream.wait_event(sync_ev[3])
-            stream.wait_event(cev[5])               # the previous G' has left
-            sn.sn_decompress_bwd(basis, Cg_rx, out=Gr)
-            cev[3].record(stream)
-            d2h_stream.wait_event(cev[3])
-            sn.sn_wire_send(Gr, Goh, stream=d2h_stream)
-            cev[5].record(d2h_stream)
+            stream.wait_event(ev["gr_free"][b_])
+            sn.sn_decompress_bwd(basis, Cg_rx, out=Grd[b_])
+            ev["gr_done"][b_].record(stream)
+            d2h_stream.wait_event(ev["gr_done"][b_])
+            sn.sn_wire_send(Grd[b_], Goh, stream=d2h_stream)
+            ev["gr_free"][b_].record(d2h_stream)
 
         for _ in range(min(args.warmup, 3)):
             e2e_step()
@@ -671,14 +686,16 @@ def run_ours(args, world, rank, local, pg):
             a.record(stream)
             for _ in range(nrep):
                 e2e_step()
-            stream.wait_stream(d2h_stream)          # the run ends when the last G' is on the host
+            stream.wait_stream(d2h_stream)          # the run ends when the last X', G' are on the host
             b.record(stream)
             b.synchronize()
             e2e_ms.append(a.elapsed_time(b) / nrep)
         sn.sn_check_errors(basis)
         e2e = max_over_ranks(pg, statistics.mean(e2e_ms), dev)
         e2e_line = {"value": world * T / (e2e / 1e3), "unit": "tokens/s",
-                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e}
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e,
+                    "pipelining": "up to two steps in flight: uploads, compute and downloads on "
+                                  "their own streams, device-side host buffers doubled"}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline and args.workload == WORKLOAD:
