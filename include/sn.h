@@ -29,7 +29,14 @@
  *     clamped: that token's output row is written as zeros and the basis'
  *     device error word records SN_ERR_BAD_ID, reported by sn_check_errors.
  *   - Only sn_basis_create allocates (and sn_basis_destroy frees); no other
- *     call allocates memory or falls back to the CPU.
+ *     call allocates memory or falls back to the CPU.  A basis holds two
+ *     scratch areas of (SM count) x 128 x (k rounded up to 16) floats that the
+ *     bf16 compress calls use for the partial sums of their last-round row
+ *     tiles: one for the forward compress calls (sn_compress_fwd,
+ *     sn_compress_fwd_projected), one for sn_compress_bwd.  Forward calls on
+ *     one basis must therefore not overlap each other in time (other streams,
+ *     other host threads), nor backward calls each other; a forward and a
+ *     backward call may.
  *   - Every wait inside a kernel is bounded; a wait that expires records
  *     SN_ERR_TIMEOUT in the error word and the kernel returns.
  */

@@ -110,6 +110,10 @@ sn_status sn_basis_create(const float *U, int32_t d, int32_t k, sn_basis_t *out,
     if (e == cudaSuccess) e = cudaMalloc(&b->ut16, sizeof(__nv_bfloat16) * (size_t)b->n_pad * d);
     if (e == cudaSuccess) e = cudaMalloc(&b->up16, sizeof(__nv_bfloat16) * (size_t)d * b->k64);
     if (e == cudaSuccess) e = cudaMalloc(&b->err, sizeof(unsigned int));
+    if (e == cudaSuccess)
+        e = cudaDeviceGetAttribute(&b->tail_cap, cudaDevAttrMultiProcessorCount, b->device);
+    for (int i = 0; i < 2 && e == cudaSuccess; ++i)
+        e = cudaMalloc(&b->tail[i], sizeof(float) * (size_t)b->tail_cap * 128 * b->n_pad);
     if (e == cudaSuccess) e = cudaMemsetAsync(b->err, 0, sizeof(unsigned int), stream);
     if (e == cudaSuccess) e = sn::prepare_basis(*b, U, stream);
     if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
@@ -131,6 +135,8 @@ sn_status sn_basis_destroy(sn_basis_t b)
     if ((e2 = cudaFree(b->ut16)) != cudaSuccess) e = e2;
     if ((e2 = cudaFree(b->up16)) != cudaSuccess) e = e2;
     if ((e2 = cudaFree(b->err)) != cudaSuccess) e = e2;
+    for (int i = 0; i < 2; ++i)
+        if ((e2 = cudaFree(b->tail[i])) != cudaSuccess) e = e2;
     delete b;
     return cuda_status(e);
 }

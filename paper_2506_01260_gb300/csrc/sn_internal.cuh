@@ -29,6 +29,11 @@ struct sn_basis {
     __nv_bfloat16 *ut16;
     __nv_bfloat16 *up16;
     unsigned int *err;
+    // fp32 partial rows of the compress contractions' split last-round tiles:
+    // [0] forward (X and projected-table modes), [1] backward; tail_cap row
+    // tiles of 128 x n_pad each (one per SM of the device)
+    float *tail[2];
+    int tail_cap;
 };
 
 namespace sn {

@@ -83,8 +83,7 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    const int nitems = p.ntiles * p.splits;
-    const int kc_total = p.nkc;
+    const int nitems = contract_items(p);
 
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
@@ -97,9 +96,8 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
         uint32_t g = 0;
         bool ok = true;
         for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x) {
-            const int tile = item / p.splits, split = item % p.splits;
-            const int kc0 = split * p.kc_per_item;
-            const int kc1 = min(kc0 + p.kc_per_item, kc_total);
+            const ItemSpan sp = item_span(p, item);
+            const int tile = sp.tile, kc0 = sp.kc0, kc1 = sp.kc1;
             const int64_t r0 = MODE == CMODE_W ? (int64_t)tile * BM
                                                : tile_row0(tile, p.reorder, p.batches, p.seq_len);
             const bool pe_tile = MODE == CMODE_X && p.has_pe && !p.has_pos &&
@@ -144,9 +142,8 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
             uint32_t g = 0, it = 0;
             bool ok = true;
             for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++it) {
-                const int split = item % p.splits;
-                const int kc0 = split * p.kc_per_item;
-                const int kc1 = min(kc0 + p.kc_per_item, kc_total);
+                const ItemSpan sp = item_span(p, item);
+                const int kc0 = sp.kc0, kc1 = sp.kc1;
                 const uint32_t b = it & 1, nb = it >> 1;
                 if (!mbar_wait(acce_b + 8 * b, (nb & 1) ^ 1, abort_flag, p.err)) {
                     ok = false;
@@ -202,10 +199,11 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
         uint32_t it = 0;
         bool ok = true;
         for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++it) {
-            const int tile = item / p.splits, split = item % p.splits;
+            const ItemSpan sp = item_span(p, item);
+            const int tile = sp.tile, split = sp.split;
             const int64_t r0 = MODE == CMODE_W ? (int64_t)tile * BM
                                                : tile_row0(tile, p.reorder, p.batches, p.seq_len);
-            if (MODE == CMODE_XP && r0 + row < p.rows) {
+            if (MODE == CMODE_XP && !sp.tail && r0 + row < p.rows) {
                 // this row's TU and PU rows are read after the item's main loop:
                 // start them towards L2 now (the epilogue warps are idle until then)
                 const int64_t t = r0 + row;
@@ -226,7 +224,24 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
             }
             tc_fence_after();
             const uint32_t taddr = tmem + b * p.acc_stride + ((uint32_t)(32 * q) << 16);
-            if (MODE == CMODE_W) {
+            if (MODE != CMODE_W && MODE != CMODE_GF && sp.tail) {
+                // a d-range of a tail tile: fp32 partial row, summed by k_sum_tail
+                float *dst = p.Ptail +
+                             (((int64_t)(tile - (p.ntiles - p.tail_tiles)) * p.tail_splits + split) *
+                                  BM + row) * p.n_pad;
+                for (int cc = 0; cc < p.n_pad / 16; ++cc) {
+                    float v[16];
+                    tmem_ld16(taddr + 16 * cc, v);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int j = 0; j < 16; j += 4)
+                        *(float4 *)(dst + 16 * cc + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0)
+                    mbar_arrive(acce_b + 8 * b);
+            } else if (MODE == CMODE_W) {
                 const int64_t c = r0 + row;
                 float *dst = p.P + ((int64_t)split * p.rows + c) * p.n_pad;
                 for (int cc = 0; cc < p.n_pad / 16; ++cc) {
@@ -317,9 +332,8 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
         uint32_t g = 0;
         bool ok = true;
         for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x) {
-            const int tile = item / p.splits, split = item % p.splits;
-            const int kc0 = split * p.kc_per_item;
-            const int kc1 = min(kc0 + p.kc_per_item, kc_total);
+            const ItemSpan sp = item_span(p, item);
+            const int tile = sp.tile, kc0 = sp.kc0, kc1 = sp.kc1;
             const int64_t r0 = tile_row0(tile, p.reorder, p.batches, p.seq_len);
             const bool pe_tile = p.has_pe && !p.has_pos && (r0 % p.seq_len) + BM <= p.seq_len;
             // element offsets of this thread's 8 rows in T_fixed and P (invalid

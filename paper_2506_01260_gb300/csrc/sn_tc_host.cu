@@ -111,14 +111,27 @@ void tile_order(int64_t T, int seq_len, bool has_pe, bool has_pos, int *reorder,
     }
 }
 
-// Split `nblk` column blocks of `ntiles` row tiles into work items so that a
-// persistent grid of `sms` CTAs sees several items each.
+// Split `nblk` column blocks of `ntiles` row tiles into work items of `bpi`
+// blocks for a persistent grid of `sms` CTAs: the longest CTA's time, counted
+// in blocks, is (rounds of the grid) x (bpi + 1), an item's start-up (its A
+// operand, the pipeline refill) costing about one block (measured on the
+// projection's third pass at W [8192, 8192]: 7 blocks per item 0.086 ms, 32
+// blocks on 128 CTAs 0.080 ms).  Among equal costs, the fewest items.
 void split_blocks(int ntiles, int nblk, int sms, int *bpi, int *chunks)
 {
-    int want = (4 * sms + ntiles - 1) / ntiles;
-    want = std::max(1, std::min(want, nblk));
-    *bpi = (nblk + want - 1) / want;
-    *chunks = (nblk + *bpi - 1) / *bpi;
+    int64_t best = -1;
+    for (int b = nblk; b >= 1; --b) {
+        const int ch = (nblk + b - 1) / b;
+        if ((nblk + ch - 1) / ch != b)
+            continue;                         // same chunk count as a larger b
+        const int64_t rounds = ((int64_t)ntiles * ch + sms - 1) / sms;
+        const int64_t cost = rounds * (b + 1);
+        if (best < 0 || cost < best) {
+            best = cost;
+            *bpi = b;
+            *chunks = ch;
+        }
+    }
 }
 
 // d-range splits of the projection's first pass: the chunk count per item that
@@ -181,6 +194,87 @@ int current_device()
 }  // namespace
 }  // namespace tc
 
+// Last-round split of the compress contractions.  With one CTA per SM a grid
+// whose last round holds rem < sms / 2 row tiles leaves most SMs idle for a
+// whole tile; those tiles instead run as s = min(4, sms / rem) items over
+// d-ranges of at least 8 chunks, writing fp32 partials to the basis' scratch,
+// and k_sum_tail adds them up (large stream: 512 tiles = 3 x 152 + 56, the
+// last round halves).  Without scratch every item is a whole tile.
+void plan_tail(tc::ContractParams &p, int sms, float *scratch, int cap)
+{
+    p.tail_tiles = 0;
+    p.tail_splits = 1;
+    p.tail_kc = p.nkc;
+    p.Ptail = nullptr;
+    const int rem = p.ntiles % sms;
+    if (!scratch || rem == 0 || p.splits != 1)
+        return;
+    const int s = std::min(std::min(4, sms / rem), p.nkc / 8);
+    if (s < 2 || rem * s > cap)
+        return;
+    const int kc = (p.nkc + s - 1) / s;
+    p.tail_tiles = rem;
+    p.tail_splits = (p.nkc + kc - 1) / kc;
+    p.tail_kc = kc;
+    p.Ptail = scratch;
+}
+
+// C rows of the split tiles: the sum of their d-range partials (minus the
+// projected embedding rows in XP mode), rounded once to bf16; a row with an
+// invalid id or position is written as zeros and flagged (X and XP modes).
+__global__ void k_sum_tail(const __grid_constant__ tc::ContractParams p, int mode)
+{
+    using namespace tc;
+    const int first = p.ntiles - p.tail_tiles;
+    const int64_t per_tile = (int64_t)BM * p.k;
+    const int64_t n = (int64_t)p.tail_tiles * per_tile;
+    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n;
+         e += (int64_t)gridDim.x * blockDim.x) {
+        const int tt = (int)(e / per_tile);
+        const int r = (int)((e / p.k) % BM);
+        const int j = (int)(e % p.k);
+        const int64_t t = tile_row0(first + tt, p.reorder, p.batches, p.seq_len) + r;
+        if (t >= p.rows)
+            continue;
+        const float *src = p.Ptail + ((int64_t)tt * p.tail_splits * BM + r) * p.n_pad + j;
+        float v = 0.f;
+        for (int sp = 0; sp < p.tail_splits; ++sp)
+            v += src[(int64_t)sp * BM * p.n_pad];
+        bool bad = false;
+        if (mode != CMODE_G) {
+            const int id = p.ids[t];
+            bad = id < 0 || id >= p.vocab;
+            int ps = 0;
+            if (p.has_pe) {
+                ps = p.has_pos ? p.pos[t] : (int)(t % p.seq_len);
+                bad = bad || ps < 0 || ps >= p.seq_len;
+            }
+            if (bad) {
+                if (j == 0)
+                    atomicOr(p.err, SN_EBIT_BAD_ID);
+            } else if (mode == CMODE_XP) {
+                v -= p.TU[(int64_t)id * p.k + j];
+                if (p.has_pe)
+                    v -= p.PU[(int64_t)ps * p.k + j];
+            }
+        }
+        p.C[t * p.k + j] = __float2bfloat16_rn(bad ? 0.f : v);
+    }
+}
+
+// The contraction over a persistent grid, then the sum of any split tiles.
+cudaError_t launch_compress(int mode, const tc::ContractParams &p, int sms, cudaStream_t s)
+{
+    using namespace tc;
+    cudaError_t e = launch_contract(mode, p, std::min(contract_items(p), sms), s);
+    if (e != cudaSuccess || p.tail_tiles == 0)
+        return e;
+    const int64_t n = (int64_t)p.tail_tiles * BM * p.k;
+    k_sum_tail<<<(int)std::min<int64_t>((n + 255) / 256, 4 * sms), 256, 0, s>>>(p, mode);
+    count_launch();
+    return cudaGetLastError();
+}
+
 cudaError_t tc_compress(const sn_basis &b, const TcArgs &a, cudaStream_t s)
 {
     using namespace tc;
@@ -217,8 +311,9 @@ cudaError_t tc_compress(const sn_basis &b, const TcArgs &a, cudaStream_t s)
     p.ntiles = (int)((a.T + BM - 1) / BM);
     tile_order(a.T, a.seq_len, has_pe, p.has_pos, &p.reorder, &p.batches);
     p.stages = contract_stages(mode, b.n_pad, b.k, has_pe);
-    const int grid = std::min(p.ntiles, sm_count(current_device()));
-    return launch_contract(mode, p, grid, s);
+    const int sms = sm_count(current_device());
+    plan_tail(p, sms, b.tail[mode == CMODE_X ? 0 : 1], b.tail_cap);
+    return launch_compress(mode, p, sms, s);
 }
 
 namespace {
@@ -282,7 +377,9 @@ cudaError_t tc_compress_projected(const sn_basis &b, const __nv_bfloat16 *X, con
     p.has_pe = PU != nullptr;
     p.has_pos = PU != nullptr && pos != nullptr;
     p.stages = contract_stages(CMODE_XP, b.n_pad, b.k, 0);
-    return launch_contract(CMODE_XP, p, std::min(p.ntiles, sm_count(current_device())), s);
+    const int sms = sm_count(current_device());
+    plan_tail(p, sms, b.tail[0], b.tail_cap);
+    return launch_compress(CMODE_XP, p, sms, s);
 }
 
 cudaError_t tc_decompress(const sn_basis &b, const TcArgs &a, __nv_bfloat16 *X_out,

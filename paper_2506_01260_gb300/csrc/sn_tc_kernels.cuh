@@ -49,7 +49,45 @@ struct ContractParams {
     int ntiles;          // row tiles
     int reorder, batches;
     int stages;
+    // X, G, XP modes: the last tail_tiles row tiles run as tail_splits items of
+    // tail_kc chunks each (the grid's last round would otherwise leave most SMs
+    // idle); those items write fp32 partial rows to Ptail
+    // [tail_tiles, tail_splits, 128, n_pad], summed afterwards by k_sum_tail
+    int tail_tiles, tail_splits, tail_kc;
+    float *Ptail;
 };
+
+// The row tile, split index and chunk range of work item `item`.
+struct ItemSpan {
+    int tile, split, kc0, kc1;
+    bool tail;
+};
+
+__host__ __device__ inline int contract_items(const ContractParams &p)
+{
+    return (p.ntiles - p.tail_tiles) * p.splits + p.tail_tiles * p.tail_splits;
+}
+
+__host__ __device__ inline ItemSpan item_span(const ContractParams &p, int item)
+{
+    ItemSpan r;
+    const int head = (p.ntiles - p.tail_tiles) * p.splits;
+    if (item < head) {
+        r.tile = item / p.splits;
+        r.split = item % p.splits;
+        r.kc0 = r.split * p.kc_per_item;
+        r.kc1 = r.kc0 + p.kc_per_item < p.nkc ? r.kc0 + p.kc_per_item : p.nkc;
+        r.tail = false;
+    } else {
+        const int j = item - head;
+        r.tile = p.ntiles - p.tail_tiles + j / p.tail_splits;
+        r.split = j % p.tail_splits;
+        r.kc0 = r.split * p.tail_kc;
+        r.kc1 = r.kc0 + p.tail_kc < p.nkc ? r.kc0 + p.tail_kc : p.nkc;
+        r.tail = true;
+    }
+    return r;
+}
 
 __host__ __device__ constexpr int contract_threads(int mode) { return mode == CMODE_X ? 320 : 192; }
 

@@ -335,3 +335,63 @@ def test_more_tiles_than_sms(sn, oracle, layout):
     # every row is covered: no row of C left at the guard fill or zero
     assert np.all(np.abs(widen(host(C))).sum(axis=1) > 0)
     basis.destroy()
+
+
+@pytest.mark.parametrize("layout", ["ragged", "few_tiles", "position_major"])
+def test_split_last_round(sn, oracle, layout):
+    """When the persistent grid's last round would hold only a few row tiles,
+    those tiles run as d-range items whose fp32 partials are summed afterwards
+    (d = 2048: 32 chunks, so 2 to 4 items a tile): a ragged last tile, fewer
+    tiles than half the SMs (every tile split), and the position-major tile
+    order.  Bad ids inside split tiles are zeroed and reported as anywhere else,
+    explicit positions are honoured, and the projected-table compress splits the
+    same way."""
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    if layout == "ragged":
+        T, n = (sms + 10) * 128 - 37, 128
+    elif layout == "few_tiles":
+        T, n = 40 * 128, 128
+    else:
+        T, n = (sms + 8) * 128, 256
+    d, k, vocab = 2048, 24, 600
+    inp = case_inputs("split_" + layout, T, n, d, k, vocab, "bf16", seed=13)
+    ids = inp["ids"].copy()
+    bad = [T - 1, T - 130, 3]
+    ids[bad] = [vocab, -1, vocab + 7]
+    basis = sn.Basis(dev(inp["U"]))
+    X, tok, pe, G = dev(inp["X"]), dev(inp["tok_emb"]), dev(inp["pos_emb"]), dev(inp["G"])
+    fullC, C = guarded((T, k), X.dtype)
+    sn.sn_compress_fwd(basis, X, dev(ids), tok, n, pos_emb=pe, out=C)
+    with pytest.raises(sn.SNError) as e:
+        sn.sn_check_errors(basis)
+    assert e.value.status == sn.SN_ERR_BAD_ID
+    fullCg, Cg = guarded((T, k), X.dtype)
+    sn.sn_compress_bwd(basis, G, out=Cg)
+    sn.sn_check_errors(basis)
+    assert guards_intact(fullC) and guards_intact(fullCg)
+    Ch = host(C)
+    assert np.all(widen(Ch[bad]) == 0)
+    _, C64, st = oracle.compress_fwd(inp["X"], ids, inp["tok_emb"], inp["U"], n,
+                                     pos_emb=inp["pos_emb"])
+    assert st == 4
+    assert rel_fro(Ch, C64) <= TOL["bf16"]
+    good = np.setdiff1d(np.arange(T), bad)
+    assert np.all(np.abs(widen(Ch[good])).sum(axis=1) > 0)
+    _, Cg64, _ = oracle.compress_bwd(inp["G"], inp["U"])
+    assert rel_fro(host(Cg), Cg64) <= TOL["bf16"]
+    # the projected-table compress over the same tiles
+    TU, PU = sn.sn_project_tables(basis, tok, pos_emb=pe)
+    Cp = sn.sn_compress_fwd_projected(basis, X, dev(ids), TU, n, PU=PU)
+    with pytest.raises(sn.SNError):
+        sn.sn_check_errors(basis)
+    assert np.all(widen(host(Cp)[bad]) == 0)
+    assert rel_fro(host(Cp), C64) <= TOL["bf16"]
+    if layout == "ragged":
+        # explicit positions (not one contiguous run per tile: gathered rows)
+        pos = np.random.default_rng(4).integers(0, n, T).astype(np.int32)
+        C = sn.sn_compress_fwd(basis, X, dev(inp["ids"]), tok, n, pos_emb=pe, pos=dev(pos))
+        sn.sn_check_errors(basis)
+        _, C64, _ = oracle.compress_fwd(inp["X"], inp["ids"], inp["tok_emb"], inp["U"], n,
+                                        pos_emb=inp["pos_emb"], pos=pos)
+        assert rel_fro(host(C), C64) <= TOL["bf16"]
+    basis.destroy()
