@@ -590,8 +590,8 @@ def run_ours(args, world, rank, local, pg):
         nxt["f2_adamw_rowconst"] = {
             "ms": ams, "algorithmic_bytes": aab, "gbs": aab / (ams / 1e3) / 1e9,
             "frac": aab / (ams / 1e3) / 1e9 / hbm, "shape": list(wo_shape),
-            "note": "fp32 W, M, V, bf16 gradient; moments + column sums of V^ (pass 1), "
-                    "W update with one rate per column (pass 2, re-reads M)"}
+            "note": "fp32 W, M, V, bf16 gradient; V + column sums of V^ (pass 1), M and W "
+                    "with one rate per column (pass 2, reads g again): 28 B moved per element"}
         del Wm, gW, Mm, Vm, aws
         nxt["f4_lossy"] = lossy_comparison(args, sn, basis, X, Xr, ids, tok, pe, n, flush,
                                            stream, hbm, pg, dev)

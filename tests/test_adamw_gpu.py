@@ -31,7 +31,7 @@ def rel(a, b):
 
 
 @pytest.mark.parametrize("gdt", ["f32", "bf16"])
-@pytest.mark.parametrize("rows,cols", [(512, 1000), (4096, 300), (7, 3)])
+@pytest.mark.parametrize("rows,cols", [(512, 1000), (4096, 300), (7, 3), (130, 1002)])
 def test_three_steps_match_oracle(sn, gdt, rows, cols):
     a = adamw_oracle()
     rng = np.random.default_rng(rows + cols)
