@@ -164,23 +164,35 @@ void project_splits(int d, int64_t m, int sms, int *splits, int *kc_per)
 size_t align256(size_t v) { return (v + 255) & ~(size_t)255; }
 
 // A^T[c, j] = sum over splits of P[split, c, j], rounded once to bf16 and
-// zero-padded to k64 columns.  One thread per output element; k64 is 64 or 128.
+// zero-padded to k64 columns.  One thread per four adjacent outputs (16-byte
+// partial loads: n_pad is a multiple of 16; an 8-byte store); k64 is 64 or 128.
 __global__ void k_sum_partials(const float *__restrict__ P, int splits, int64_t m, int n_pad,
                                int k, int k64_log2, __nv_bfloat16 *__restrict__ At)
 {
-    const int64_t n = m << k64_log2;
+    const int64_t n = m << (k64_log2 - 2);
     const int64_t split_stride = m * n_pad;
+    const int q_log2 = k64_log2 - 2;
     for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n;
          e += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t c = e >> k64_log2;
-        const int j = (int)(e & ((1 << k64_log2) - 1));
-        float s = 0.f;
+        const int64_t c = e >> q_log2;
+        const int j = 4 * (int)(e & ((1 << q_log2) - 1));
+        float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
         if (j < k) {
             const float *src = P + c * n_pad + j;
-            for (int sp = 0; sp < splits; ++sp, src += split_stride)
-                s += __ldg(src);
+            for (int sp = 0; sp < splits; ++sp, src += split_stride) {
+                const float4 v = __ldg((const float4 *)src);
+                s.x += v.x;
+                s.y += v.y;
+                s.z += v.z;
+                s.w += v.w;
+            }
         }
-        At[e] = __float2bfloat16_rn(s);
+        __nv_bfloat162 lo = __floats2bfloat162_rn(j < k ? s.x : 0.f, j + 1 < k ? s.y : 0.f);
+        __nv_bfloat162 hi = __floats2bfloat162_rn(j + 2 < k ? s.z : 0.f, j + 3 < k ? s.w : 0.f);
+        uint2 out;
+        out.x = *(const uint32_t *)&lo;
+        out.y = *(const uint32_t *)&hi;
+        *(uint2 *)(At + (c << k64_log2) + j) = out;
     }
 }
 
@@ -571,7 +583,11 @@ cudaError_t tc_project(const sn_basis &b, const __nv_bfloat16 *W, int64_t cols, 
     if (e != cudaSuccess)
         return e;
     // pass 2: sum the partials, round A^T to bf16 [cols, k64] (zero-padded)
-    k_sum_partials<<<4 * sms, 256, 0, s>>>(P, splits, cols, b.n_pad, b.k, b.k64 == 64 ? 6 : 7, At);
+    {
+        const int64_t n4 = cols * (b.k64 / 4);
+        k_sum_partials<<<(int)std::min<int64_t>((n4 + 255) / 256, 4 * sms), 256, 0, s>>>(
+            P, splits, cols, b.n_pad, b.k, b.k64 == 64 ? 6 : 7, At);
+    }
     count_launch();
     if ((e = cudaGetLastError()) != cudaSuccess)
         return e;
