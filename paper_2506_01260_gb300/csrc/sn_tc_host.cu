@@ -234,43 +234,40 @@ void plan_tail(tc::ContractParams &p, int sms, float *scratch, int cap)
 // C rows of the split tiles: the sum of their d-range partials (minus the
 // projected embedding rows in XP mode), rounded once to bf16; a row with an
 // invalid id or position is written as zeros and flagged (X and XP modes).
-__global__ void k_sum_tail(const __grid_constant__ tc::ContractParams p, int mode)
+// Grid (tail tiles, 128 / 8): one warp per row, the lanes across its k columns.
+__global__ void __launch_bounds__(256) k_sum_tail(const __grid_constant__ tc::ContractParams p,
+                                                  int mode)
 {
     using namespace tc;
-    const int first = p.ntiles - p.tail_tiles;
-    const int64_t per_tile = (int64_t)BM * p.k;
-    const int64_t n = (int64_t)p.tail_tiles * per_tile;
-    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n;
-         e += (int64_t)gridDim.x * blockDim.x) {
-        const int tt = (int)(e / per_tile);
-        const int r = (int)((e / p.k) % BM);
-        const int j = (int)(e % p.k);
-        const int64_t t = tile_row0(first + tt, p.reorder, p.batches, p.seq_len) + r;
-        if (t >= p.rows)
-            continue;
-        const float *src = p.Ptail + ((int64_t)tt * p.tail_splits * BM + r) * p.n_pad + j;
+    const int tt = blockIdx.x;
+    const int r = 8 * blockIdx.y + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+    const int64_t row = tile_row0(p.ntiles - p.tail_tiles + tt, p.reorder, p.batches, p.seq_len) + r;
+    if (row >= p.rows)
+        return;
+    bool bad = false;
+    int id = 0, ps = 0;
+    if (mode != CMODE_G) {
+        id = p.ids[row];
+        bad = id < 0 || id >= p.vocab;
+        if (p.has_pe) {
+            ps = p.has_pos ? p.pos[row] : (int)(row % p.seq_len);
+            bad = bad || ps < 0 || ps >= p.seq_len;
+        }
+        if (bad && lane == 0)
+            atomicOr(p.err, SN_EBIT_BAD_ID);
+    }
+    const float *src = p.Ptail + ((int64_t)tt * p.tail_splits * BM + r) * p.n_pad;
+    const int64_t split_stride = (int64_t)BM * p.n_pad;
+    for (int j = lane; j < p.k; j += 32) {
         float v = 0.f;
         for (int sp = 0; sp < p.tail_splits; ++sp)
-            v += src[(int64_t)sp * BM * p.n_pad];
-        bool bad = false;
-        if (mode != CMODE_G) {
-            const int id = p.ids[t];
-            bad = id < 0 || id >= p.vocab;
-            int ps = 0;
-            if (p.has_pe) {
-                ps = p.has_pos ? p.pos[t] : (int)(t % p.seq_len);
-                bad = bad || ps < 0 || ps >= p.seq_len;
-            }
-            if (bad) {
-                if (j == 0)
-                    atomicOr(p.err, SN_EBIT_BAD_ID);
-            } else if (mode == CMODE_XP) {
-                v -= p.TU[(int64_t)id * p.k + j];
-                if (p.has_pe)
-                    v -= p.PU[(int64_t)ps * p.k + j];
-            }
+            v += src[sp * split_stride + j];
+        if (!bad && mode == CMODE_XP) {
+            v -= p.TU[(int64_t)id * p.k + j];
+            if (p.has_pe)
+                v -= p.PU[(int64_t)ps * p.k + j];
         }
-        p.C[t * p.k + j] = __float2bfloat16_rn(bad ? 0.f : v);
+        p.C[row * p.k + j] = __float2bfloat16_rn(bad ? 0.f : v);
     }
 }
 
@@ -281,8 +278,7 @@ cudaError_t launch_compress(int mode, const tc::ContractParams &p, int sms, cuda
     cudaError_t e = launch_contract(mode, p, std::min(contract_items(p), sms), s);
     if (e != cudaSuccess || p.tail_tiles == 0)
         return e;
-    const int64_t n = (int64_t)p.tail_tiles * BM * p.k;
-    k_sum_tail<<<(int)std::min<int64_t>((n + 255) / 256, 4 * sms), 256, 0, s>>>(p, mode);
+    k_sum_tail<<<dim3(p.tail_tiles, BM / 8), 256, 0, s>>>(p, mode);
     count_launch();
     return cudaGetLastError();
 }
