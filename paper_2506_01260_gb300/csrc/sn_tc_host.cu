@@ -452,32 +452,42 @@ namespace tc {
 namespace {
 
 // CgT[j, t] = Cg[t, j] for j < k, t < T; zero for k <= j < n_pad and T <= t < Tp.
-__global__ void k_transpose_pad(const __nv_bfloat16 *__restrict__ Cg, int64_t T, int k, int n_pad,
-                                int64_t Tp, __nv_bfloat16 *__restrict__ CgT)
+__global__ void __launch_bounds__(256) k_transpose_pad(const __nv_bfloat16 *__restrict__ Cg, int64_t T,
+                                                      int k, int n_pad, int64_t Tp,
+                                                      __nv_bfloat16 *__restrict__ CgT)
 {
-    const int64_t n = (int64_t)n_pad * Tp;
-    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n;
-         e += (int64_t)gridDim.x * blockDim.x) {
-        const int j = (int)(e / Tp);
-        const int64_t t = e - (int64_t)j * Tp;
-        CgT[e] = (j < k && t < T) ? Cg[t * k + j] : __float2bfloat16_rn(0.f);
+    // 64 tokens per block through shared memory: their k-wide rows are one
+    // contiguous run of Cg (coalesced reads), each output row j gets 64
+    // consecutive tokens (128-byte writes); the row pitch of 130 elements keeps
+    // the column reads on distinct banks.  k <= 128.
+    __shared__ __nv_bfloat16 tile[64][130];
+    const int64_t t0 = (int64_t)blockIdx.x * 64;
+    const int nt = (int)(T - t0 < 64 ? (T - t0 > 0 ? T - t0 : 0) : 64);
+    for (int f = threadIdx.x; f < 64 * k; f += blockDim.x) {
+        const int tl = f / k, j = f - tl * k;
+        tile[tl][j] = tl < nt ? Cg[t0 * k + f] : __float2bfloat16_rn(0.f);
+    }
+    __syncthreads();
+    for (int f = threadIdx.x; f < n_pad * 64; f += blockDim.x) {
+        const int j = f >> 6, t = f & 63;
+        CgT[(int64_t)j * Tp + t0 + t] = j < k ? tile[t][j] : __float2bfloat16_rn(0.f);
     }
 }
 
 // M[i, j] += sum over splits of P[split, i, j], j < k (M row-major [d, k]).
-__global__ void k_accumulate_partials(const float *__restrict__ P, int splits, int64_t d,
-                                      int n_pad, int k, float *__restrict__ M)
+__global__ void __launch_bounds__(256) k_accumulate_partials(const float *__restrict__ P, int splits,
+                                                            int64_t d, int n_pad, int k,
+                                                            float *__restrict__ M)
 {
-    const int64_t n = d * k;
-    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n;
-         e += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t i = e / k;
-        const int j = (int)(e - i * k);
-        float s = 0.f;
-        for (int sp = 0; sp < splits; ++sp)
-            s += __ldg(P + ((int64_t)sp * d + i) * n_pad + j);
-        M[e] += s;
-    }
+    // two rows of M per block, one thread per column (k <= 128)
+    const int64_t i = 2 * (int64_t)blockIdx.x + (threadIdx.x >> 7);
+    const int j = threadIdx.x & 127;
+    if (i >= d || j >= k)
+        return;
+    float s = 0.f;
+    for (int sp = 0; sp < splits; ++sp)
+        s += __ldg(P + ((int64_t)sp * d + i) * n_pad + j);
+    M[i * k + j] += s;
 }
 
 }  // namespace
@@ -507,7 +517,7 @@ cudaError_t tc_grassmann_accumulate(const sn_basis &b, const __nv_bfloat16 *G,
     float *P = (float *)((char *)workspace +
                          align256(sizeof(__nv_bfloat16) * (size_t)b.n_pad * Tp));
     // Cg^T, K-major over the tokens: the B operand of M = G^T Cg
-    k_transpose_pad<<<4 * sms, 256, 0, s>>>(Cg, T, b.k, b.n_pad, Tp, CgT);
+    k_transpose_pad<<<(unsigned)(Tp / 64), 256, 0, s>>>(Cg, T, b.k, b.n_pad, Tp, CgT);
     count_launch();
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess)
@@ -538,7 +548,7 @@ cudaError_t tc_grassmann_accumulate(const sn_basis &b, const __nv_bfloat16 *G,
     e = launch_contract(CMODE_W, p, std::min(p.ntiles * splits, sms), s);
     if (e != cudaSuccess)
         return e;
-    k_accumulate_partials<<<4 * sms, 256, 0, s>>>(P, splits, b.d, b.n_pad, b.k, M);
+    k_accumulate_partials<<<(unsigned)((b.d + 1) / 2), 256, 0, s>>>(P, splits, b.d, b.n_pad, b.k, M);
     count_launch();
     return cudaGetLastError();
 }
