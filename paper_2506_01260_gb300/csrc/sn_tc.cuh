@@ -330,6 +330,17 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
     return r;
 }
 
+// Programmatic dependent launch: a kernel launched with programmatic stream
+// serialization may start before the previous kernel of its stream ends;
+// griddep_wait blocks until that kernel has completed and its writes are
+// visible (a no-op for a kernel launched normally), griddep_launch_dependents
+// lets the next such kernel start being scheduled.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch_dependents()
+{
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // Prefetch the 128-byte lines of [p, p + bytes) into L2.
 __device__ __forceinline__ void prefetch_l2_range(const void *p, int bytes)
 {

@@ -82,6 +82,8 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    griddep_launch_dependents();   // a dependent launch may be scheduled now
+    griddep_wait();                // launched as a dependent: the previous kernel's writes
 
     const int nitems = contract_items(p);
 
@@ -387,27 +389,43 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
 namespace {
 
 template <int MODE>
-cudaError_t launch_mode(const ContractParams &p, int grid, uint32_t smem, cudaStream_t s)
+cudaError_t launch_mode(const ContractParams &p, int grid, uint32_t smem, cudaStream_t s,
+                        bool dependent)
 {
     cudaError_t e =
         cudaFuncSetAttribute(k_contract<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e == cudaSuccess)
+    if (e != cudaSuccess)
+        return e;
+    if (!dependent) {
         k_contract<MODE><<<grid, contract_threads(MODE), smem, s>>>(p);
-    return e;
+        return e;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(contract_threads(MODE));
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, k_contract<MODE>, p);
 }
 
 }  // namespace
 
-cudaError_t launch_contract(int mode, const ContractParams &p, int grid, cudaStream_t s)
+cudaError_t launch_contract(int mode, const ContractParams &p, int grid, cudaStream_t s,
+                            bool dependent)
 {
     const ContractPlan pl = contract_plan(mode, p.n_pad, p.k, p.has_pe, p.stages);
     cudaError_t e;
     switch (mode) {
-    case CMODE_X: e = launch_mode<CMODE_X>(p, grid, pl.total, s); break;
-    case CMODE_G: e = launch_mode<CMODE_G>(p, grid, pl.total, s); break;
-    case CMODE_W: e = launch_mode<CMODE_W>(p, grid, pl.total, s); break;
-    case CMODE_GF: e = launch_mode<CMODE_GF>(p, grid, pl.total, s); break;
-    default: e = launch_mode<CMODE_XP>(p, grid, pl.total, s); break;
+    case CMODE_X: e = launch_mode<CMODE_X>(p, grid, pl.total, s, dependent); break;
+    case CMODE_G: e = launch_mode<CMODE_G>(p, grid, pl.total, s, dependent); break;
+    case CMODE_W: e = launch_mode<CMODE_W>(p, grid, pl.total, s, dependent); break;
+    case CMODE_GF: e = launch_mode<CMODE_GF>(p, grid, pl.total, s, dependent); break;
+    default: e = launch_mode<CMODE_XP>(p, grid, pl.total, s, dependent); break;
     }
     if (e != cudaSuccess)
         return e;

@@ -82,6 +82,7 @@ __global__ void __launch_bounds__(kExpandThreads, 1) k_expand(const __grid_const
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    griddep_wait();   // the projection's third pass: the previous passes' writes are visible
     const int nitems = p.ntiles * p.chunks;
 
     if (warp == 0) {
@@ -305,7 +306,8 @@ __global__ void __launch_bounds__(kExpandThreads, 1) k_expand(const __grid_const
 
 }  // namespace
 
-cudaError_t launch_expand(int amode, const ExpandParams &p, int grid, cudaStream_t s)
+cudaError_t launch_expand(int amode, const ExpandParams &p, int grid, cudaStream_t s,
+                          bool dependent)
 {
     const ExpandPlan pl = expand_plan(p.katoms, p.stages);
     cudaError_t e;
@@ -317,8 +319,23 @@ cudaError_t launch_expand(int amode, const ExpandParams &p, int grid, cudaStream
     } else {
         e = cudaFuncSetAttribute(k_expand<AMODE_TMA>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  pl.total);
-        if (e == cudaSuccess)
+        if (e == cudaSuccess && dependent) {
+            // may start while the previous kernel of the stream finishes (it
+            // waits for it in griddep_wait before touching global memory)
+            cudaLaunchConfig_t cfg = {};
+            cfg.gridDim = dim3(grid);
+            cfg.blockDim = dim3(kExpandThreads);
+            cfg.dynamicSmemBytes = pl.total;
+            cfg.stream = s;
+            cudaLaunchAttribute attr[1];
+            attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+            attr[0].val.programmaticStreamSerializationAllowed = 1;
+            cfg.attrs = attr;
+            cfg.numAttrs = 1;
+            e = cudaLaunchKernelEx(&cfg, k_expand<AMODE_TMA>, p);
+        } else if (e == cudaSuccess) {
             k_expand<AMODE_TMA><<<grid, kExpandThreads, pl.total, s>>>(p);
+        }
     }
     if (e != cudaSuccess)
         return e;

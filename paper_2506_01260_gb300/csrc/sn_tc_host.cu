@@ -6,6 +6,7 @@
 #include <cstring>
 #include <mutex>
 
+#include "sn_tc.cuh"
 #include "sn_tc_kernels.cuh"
 
 namespace sn {
@@ -163,12 +164,32 @@ void project_splits(int d, int64_t m, int sms, int *splits, int *kc_per)
 
 size_t align256(size_t v) { return (v + 255) & ~(size_t)255; }
 
+// Launch `kernel` so that it may start while the previous kernel of the
+// stream finishes; the kernel waits for it in griddep_wait.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_dependent(void (*kernel)(KArgs...), dim3 grid, dim3 block, cudaStream_t s,
+                             Args... args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 // A^T[c, j] = sum over splits of P[split, c, j], rounded once to bf16 and
 // zero-padded to k64 columns.  One thread per four adjacent outputs (16-byte
 // partial loads: n_pad is a multiple of 16; an 8-byte store); k64 is 64 or 128.
 __global__ void k_sum_partials(const float *__restrict__ P, int splits, int64_t m, int n_pad,
                                int k, int k64_log2, __nv_bfloat16 *__restrict__ At)
 {
+    griddep_wait();                   // the first pass's partials are visible
+    griddep_launch_dependents();
     const int64_t n = m << (k64_log2 - 2);
     const int64_t split_stride = m * n_pad;
     const int q_log2 = k64_log2 - 2;
@@ -239,6 +260,7 @@ __global__ void __launch_bounds__(256) k_sum_tail(const __grid_constant__ tc::Co
                                                   int mode)
 {
     using namespace tc;
+    griddep_wait();                   // the contraction's partials are visible
     const int tt = blockIdx.x;
     const int r = 8 * blockIdx.y + (threadIdx.x >> 5), lane = threadIdx.x & 31;
     const int64_t row = tile_row0(p.ntiles - p.tail_tiles + tt, p.reorder, p.batches, p.seq_len) + r;
@@ -278,9 +300,9 @@ cudaError_t launch_compress(int mode, const tc::ContractParams &p, int sms, cuda
     cudaError_t e = launch_contract(mode, p, std::min(contract_items(p), sms), s);
     if (e != cudaSuccess || p.tail_tiles == 0)
         return e;
-    k_sum_tail<<<dim3(p.tail_tiles, BM / 8), 256, 0, s>>>(p, mode);
+    e = launch_dependent(k_sum_tail, dim3(p.tail_tiles, BM / 8), dim3(256), s, p, mode);
     count_launch();
-    return cudaGetLastError();
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t tc_compress(const sn_basis &b, const TcArgs &a, cudaStream_t s)
@@ -479,6 +501,7 @@ __global__ void __launch_bounds__(256) k_accumulate_partials(const float *__rest
                                                             int64_t d, int n_pad, int k,
                                                             float *__restrict__ M)
 {
+    griddep_wait();                   // the contraction's partials are visible
     // two rows of M per block, one thread per column (k <= 128)
     const int64_t i = 2 * (int64_t)blockIdx.x + (threadIdx.x >> 7);
     const int j = threadIdx.x & 127;
@@ -545,12 +568,13 @@ cudaError_t tc_grassmann_accumulate(const sn_basis &b, const __nv_bfloat16 *G,
     p.splits = splits;
     p.ntiles = (b.d + BM - 1) / BM;
     p.stages = contract_stages(CMODE_W, b.n_pad, b.k, 0);
-    e = launch_contract(CMODE_W, p, std::min(p.ntiles * splits, sms), s);
+    e = launch_contract(CMODE_W, p, std::min(p.ntiles * splits, sms), s, true);
     if (e != cudaSuccess)
         return e;
-    k_accumulate_partials<<<(unsigned)((b.d + 1) / 2), 256, 0, s>>>(P, splits, b.d, b.n_pad, b.k, M);
+    e = launch_dependent(k_accumulate_partials, dim3((unsigned)((b.d + 1) / 2)), dim3(256), s,
+                         (const float *)P, splits, (int64_t)b.d, b.n_pad, b.k, M);
     count_launch();
-    return cudaGetLastError();
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t tc_project(const sn_basis &b, const __nv_bfloat16 *W, int64_t cols, int64_t ld,
@@ -590,9 +614,13 @@ cudaError_t tc_project(const sn_basis &b, const __nv_bfloat16 *W, int64_t cols, 
         return e;
     // pass 2: sum the partials, round A^T to bf16 [cols, k64] (zero-padded)
     {
+        // launched to start while the first pass finishes (it waits for it)
         const int64_t n4 = cols * (b.k64 / 4);
-        k_sum_partials<<<(int)std::min<int64_t>((n4 + 255) / 256, 4 * sms), 256, 0, s>>>(
-            P, splits, cols, b.n_pad, b.k, b.k64 == 64 ? 6 : 7, At);
+        e = launch_dependent(k_sum_partials, dim3((unsigned)std::min<int64_t>((n4 + 255) / 256, 4 * sms)),
+                             dim3(256), s, (const float *)P, splits, cols, b.n_pad, b.k,
+                             b.k64 == 64 ? 6 : 7, At);
+        if (e != cudaSuccess)
+            return e;
     }
     count_launch();
     if ((e = cudaGetLastError()) != cudaSuccess)
@@ -622,7 +650,7 @@ cudaError_t tc_project(const sn_basis &b, const __nv_bfloat16 *W, int64_t cols, 
     q.ntiles = (b.d + BM - 1) / BM;
     split_blocks(q.ntiles, q.nblk, sms, &q.bpi, &q.chunks);
     q.stages = expand_stages(q.katoms);
-    return launch_expand(AMODE_TMA, q, std::min(q.ntiles * q.chunks, sms), s);
+    return launch_expand(AMODE_TMA, q, std::min(q.ntiles * q.chunks, sms), s, true);
 }
 
 }  // namespace sn

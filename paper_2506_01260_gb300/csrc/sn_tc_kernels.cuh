@@ -209,8 +209,10 @@ __host__ __device__ inline int64_t tile_row0(int tile, int reorder, int batches,
 }
 
 // ---- host side -----------------------------------------------------------------------
-cudaError_t launch_contract(int mode, const ContractParams &p, int grid, cudaStream_t s);
-cudaError_t launch_expand(int amode, const ExpandParams &p, int grid, cudaStream_t s);
+cudaError_t launch_contract(int mode, const ContractParams &p, int grid, cudaStream_t s,
+                            bool dependent = false);
+cudaError_t launch_expand(int amode, const ExpandParams &p, int grid, cudaStream_t s,
+                          bool dependent = false);
 cudaError_t launch_reconstruct(const ExpandParams &p, int grid, cudaStream_t s);
 
 }  // namespace tc
