@@ -188,6 +188,26 @@ def test_project_weight(sn, oracle, dtype, d, k, cols, ld):
     basis.destroy()
 
 
+@pytest.mark.parametrize("d,k,cols", [(8192, 82, 8192), (4096, 41, 14336)])
+def test_project_weight_in_place_full_size(sn, d, k, cols):
+    """At the benchmark's weight shapes the projection's three passes overlap
+    their neighbours' start-up (programmatic dependent launch); projecting in
+    place must give exactly the out-of-place result, so no pass may write W'
+    before the first pass has read all of W."""
+    rng = np.random.default_rng(d + cols)
+    U = W.orthonormal_basis(d, k, rng).astype(np.float32)
+    basis = sn.Basis(dev(U))
+    g = torch.Generator(device="cuda").manual_seed(3)
+    Wd = (0.02 * torch.randn(d, cols, generator=g, device="cuda")).to(torch.bfloat16)
+    ref = sn.sn_project_weight(basis, Wd)
+    for _ in range(3):
+        Wi = Wd.clone()
+        sn.sn_project_weight(basis, Wi, out=Wi)
+        sn.sn_check_errors(basis)
+        assert torch.equal(Wi, ref)
+    basis.destroy()
+
+
 @pytest.mark.parametrize("dtype", DTYPES)
 def test_projection_identities(sn, dtype):
     """P^2 = P and P U = U on the GPU output (Sec. 4.3; U^T U = I, App. A)."""
