@@ -210,7 +210,8 @@ sn_status sn_grassmann_residual(sn_basis_t basis, sn_dtype dtype, const void *G,
                                 int64_t T, double *acc, sn_stream_t stream);
 
 /* U_new = Q of U - eta * tangent(-2 M / K), the QR factor with diag(R) > 0
- * (CholeskyQR2 with fp64 Gram matrices).  M: fp32 [d, k] from
+ * (CholeskyQR2 in fp32, Gram matrices summed over row blocks in fp64; U_new^T
+ * U_new = I to about 1e-7 for a step within reach of the identity).  M: fp32 [d, k] from
  * sn_grassmann_accumulate over K >= 1 iterations; U_new: fp32 [d, k], may not
  * overlap M.  A non-positive pivot records SN_ERR_NUMERIC for sn_check_errors. */
 sn_status sn_grassmann_step(sn_basis_t basis, const float *M, int32_t K, float eta, float *U_new,

@@ -34,8 +34,10 @@ def _free_port():
 
 
 def _worker(rank, world, port, outdir):
+    # CPU ranks (gloo) even on a machine with a GPU: the bench's set-up picks
+    # NCCL whenever CUDA is visible
     os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), WORLD_SIZE=str(world),
-                      RANK=str(rank), LOCAL_RANK=str(rank))
+                      RANK=str(rank), LOCAL_RANK=str(rank), CUDA_VISIBLE_DEVICES="")
     sys.path.insert(0, ROOT)
     import torch
     bench = _load("bench_under_test", os.path.join(ROOT, "bench.py"))
