@@ -188,17 +188,33 @@ __global__ void __launch_bounds__(128) k_cholesky_inv(const float *__restrict__ 
 __global__ void k_residual(const __nv_bfloat16 *__restrict__ G, int64_t ng,
                            const __nv_bfloat16 *__restrict__ Cg, int64_t nc, double *acc)
 {
+    // squares summed in fp32 over 16 chunks of 8 (128 positive terms) at a
+    // time, then into fp64: this GPU's fp64 rate could not keep up with one
+    // fp64 operation per element
     double s = 0.0;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     const int64_t t0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    for (int64_t e = t0; e < ng / 8; e += stride) {
-        const uint4 w = __ldg((const uint4 *)G + e);
-        const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+    const int64_t n8 = ng / 8;
+    for (int64_t e0 = t0; e0 < n8; e0 += 16 * stride) {
+        float f = 0.f;
+        for (int64_t e1 = e0; e1 < e0 + 16 * stride && e1 < n8; e1 += 4 * stride) {
+            uint4 w[4];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const float lo = __uint_as_float(ws[q] << 16), hi = __uint_as_float(ws[q] & 0xFFFF0000u);
-            s += (double)lo * lo + (double)hi * hi;
+            for (int u = 0; u < 4; ++u)     // four 16-byte loads in flight
+                w[u] = e1 + u * stride < n8 ? __ldg((const uint4 *)G + e1 + u * stride)
+                                            : make_uint4(0, 0, 0, 0);
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const uint32_t ws[4] = {w[u].x, w[u].y, w[u].z, w[u].w};
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float lo = __uint_as_float(ws[q] << 16);
+                    const float hi = __uint_as_float(ws[q] & 0xFFFF0000u);
+                    f = fmaf(lo, lo, fmaf(hi, hi, f));
+                }
+            }
         }
+        s += (double)f;
     }
     for (int64_t e = (ng / 8) * 8 + t0; e < ng; e += stride) {
         const float v = __bfloat162float(G[e]);
