@@ -54,7 +54,7 @@ typedef enum {
     SN_OK = 0,
     SN_ERR_INVALID_ARG = 1,   /* bad size, NULL pointer, k > d, overlap, ... */
     SN_ERR_ALIGNMENT = 2,     /* a pointer or leading dimension breaks the 16-byte rule */
-    SN_ERR_UNSUPPORTED = 3,   /* valid request this build does not implement */
+    SN_ERR_UNSUPPORTED = 3,   /* valid request the library does not implement */
     SN_ERR_BAD_ID = 4,        /* asynchronous: an id or position was out of range */
     SN_ERR_TIMEOUT = 5,       /* asynchronous: a bounded in-kernel wait expired */
     SN_ERR_CUDA = 6,          /* a CUDA runtime call failed */
