@@ -278,6 +278,19 @@ sn_status sn_wire_recv(const void *src_host, void *dst_device, size_t bytes, sn_
  * (SN_ERR_BAD_ID or SN_ERR_TIMEOUT; SN_OK if none was recorded). */
 sn_status sn_check_errors(sn_basis_t basis, sn_stream_t stream);
 
+/* Failure-detection self-test of the bounded-wait rule: every in-kernel wait
+ * (mbarrier phases, copies, MMA commits) gives up after a fixed limit of 2 s
+ * instead of hanging.  Launches on `stream` one CTA of two warps that sets up
+ * like the pipeline kernels (an mbarrier, an abort flag, 32 columns of tensor
+ * memory) and waits for a barrier phase that nothing ever completes, with the
+ * same bounded wait.  The first warp past the limit records SN_ERR_TIMEOUT in
+ * the basis' error word and raises the abort flag, the other stops on the flag,
+ * and the CTA frees its tensor memory and returns.  Asynchronous: the next
+ * sn_check_errors on the basis returns SN_ERR_TIMEOUT; the basis and the CUDA
+ * context stay usable.  Errors: SN_ERR_INVALID_ARG (null basis, basis of
+ * another device), SN_ERR_CUDA (launch failure). */
+sn_status sn_selftest_wait_timeout(sn_basis_t basis, sn_stream_t stream);
+
 /* Number of kernels this library has launched in this process. */
 uint64_t sn_launch_count(void);
 

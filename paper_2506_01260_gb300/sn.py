@@ -63,6 +63,7 @@ _sig("sn_wire_bytes", [_P, _ST, _I64, ctypes.POINTER(_SZ)])
 _sig("sn_wire_send", [_P, _P, _SZ, _P])
 _sig("sn_wire_recv", [_P, _P, _SZ, _P])
 _sig("sn_check_errors", [_P, _P])
+_sig("sn_selftest_wait_timeout", [_P, _P])
 _sig("sn_launch_count", [], ctypes.c_uint64)
 _sig("sn_status_string", [_ST], ctypes.c_char_p)
 
@@ -75,7 +76,8 @@ EXPORTS = ["sn_basis_create", "sn_basis_destroy", "sn_basis_shape", "sn_compress
            "sn_grassmann_step", "sn_adamw_rowconst", "sn_topk_compress", "sn_topk_restore",
            "sn_sign_compress", "sn_sign_restore",
            "sn_wire_bytes", "sn_wire_send",
-           "sn_wire_recv", "sn_check_errors", "sn_launch_count", "sn_status_string"]
+           "sn_wire_recv", "sn_check_errors", "sn_selftest_wait_timeout", "sn_launch_count",
+           "sn_status_string"]
 
 
 class SNError(RuntimeError):
@@ -507,6 +509,14 @@ def sn_wire_recv(src_host, dst_device, stream=None):
 def sn_check_errors(basis, stream=None):
     """Synchronise the stream; raise SNError if a bad id or a timeout was recorded."""
     _check(_lib.sn_check_errors(basis.handle, _stream(stream)), "sn_check_errors")
+
+
+def sn_selftest_wait_timeout(basis, stream=None):
+    """Launch the bounded-wait self-test: one CTA waits on a barrier nothing
+    completes, gives up after the library's wait limit (2 s) and records
+    SN_ERR_TIMEOUT for the next sn_check_errors."""
+    _check(_lib.sn_selftest_wait_timeout(basis.handle, _stream(stream)),
+           "sn_selftest_wait_timeout")
 
 
 def sn_launch_count():
