@@ -295,9 +295,10 @@ def lossy_comparison(args, sn, basis, X, Xr, ids, tok, pe, n, flush, stream, hbm
     of the lossy comparators on the same activation batch, with the wire bytes of
     each: top-k at the codec's wire size (kk = k / 2: a bf16 value and a 16-bit
     column per kept entry), sign quantization (1 bit per entry, the smallest
-    quantizer) and the randomized rank-r factorisation of the whole batch at the
-    codec's wire size (r = T k / (T + d)).  Top-k and sign are timed like the
-    step's kernels."""
+    quantizer), row-scaled int8 and fp8 e4m3 quantization (8 bits per entry)
+    and the randomized rank-r factorisation of the whole batch at the
+    codec's wire size (r = T k / (T + d)).  Top-k, sign and the 8-bit
+    quantizers are timed like the step's kernels."""
     import torch
     from paper_2506_01260_gb300 import comparators
 
@@ -346,6 +347,18 @@ def lossy_comparison(args, sn, basis, X, Xr, ids, tok, pe, n, flush, stream, hbm
                    "compress_gbs": sab / (sms / 1e3) / 1e9,
                    "compress_frac": sab / (sms / 1e3) / 1e9 / hbm}
     del Xh, bits, scale
+    codes = torch.empty(T, d, dtype=torch.uint8, device=dev)
+    qscale = torch.empty(T, dtype=torch.float32, device=dev)
+    qab = 2 * T * d + T * d + 4 * T
+    for fmt in ("int8", "e4m3"):
+        qms = timed(lambda: sn.sn_quant_compress(X, fmt, codes=codes, scale=qscale),
+                    min(args.steps, 20))
+        Xh, wb = comparators.quant_roundtrip(X, fmt)
+        out[fmt] = {"wire_bytes": wb, "rel_error": rel(Xh), "compress_ms": qms,
+                    "compress_gbs": qab / (qms / 1e3) / 1e9,
+                    "compress_frac": qab / (qms / 1e3) / 1e9 / hbm}
+        del Xh
+    del codes, qscale
     r = T * k // (T + d)
     Xh, wb = comparators.lowrank_roundtrip(X, r)
     out["lowrank"] = {"r": r, "wire_bytes": wb, "rel_error": rel(Xh)}

@@ -263,6 +263,26 @@ sn_status sn_sign_compress(const void *X, int64_t T, int32_t d, uint32_t *bits, 
 sn_status sn_sign_restore(const uint32_t *bits, const float *scale, int64_t T, int32_t d,
                           void *X_out, sn_stream_t stream);
 
+/* Row-scaled 8-bit quantization, the comparison's quantizer at twice the
+ * rate of the 1-bit one's bits per entry (X finite).  Per row t:
+ * a = max |X[t, :]|, scale[t] = a / qmax (fp32), codes[t, c] = Q(X[t, c] * r)
+ * with r = qmax / a (0 for a zero row), both fp32 operations.
+ *   SN_Q_INT8  qmax = 127, Q = round half to even, clamp to [-127, 127],
+ *              codes are int8 two's complement;
+ *   SN_Q_E4M3  qmax = 448, Q = nearest fp8 e4m3 value (1-4-3, bias 7), ties to
+ *              even, magnitudes past 448 saturate to 448, sign kept.
+ * codes: uint8 [T, d] row-major (8-byte aligned), scale: fp32 [T]; T * d + 4 T
+ * bytes on the wire, half of bf16.  Errors: SN_ERR_INVALID_ARG (format, sizes,
+ * null or overlapping buffers), SN_ERR_ALIGNMENT. */
+typedef enum { SN_Q_INT8 = 0, SN_Q_E4M3 = 1 } sn_qformat;
+sn_status sn_quant_compress(const void *X, int64_t T, int32_t d, int32_t format, uint8_t *codes,
+                            float *scale, sn_stream_t stream);
+
+/* X_out[t, c] = decode(codes[t, c]) * scale[t], the product in fp32 rounded
+ * once to bf16. */
+sn_status sn_quant_restore(const uint8_t *codes, const float *scale, int64_t T, int32_t d,
+                           int32_t format, void *X_out, sn_stream_t stream);
+
 /* Bytes on the wire for T tokens: T * k * element size (Sec. 4.3: k/d of X). */
 sn_status sn_wire_bytes(sn_basis_t basis, sn_dtype dtype, int64_t T, size_t *bytes);
 

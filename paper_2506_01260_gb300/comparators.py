@@ -30,6 +30,14 @@ def sign_roundtrip(X):
     return sn.sn_sign_restore(bits, scale, d), T * ((d + 7) // 8) + 4 * T
 
 
+def quant_roundtrip(X, fmt):
+    """Row-scaled 8-bit round trip ("int8" or "e4m3"): T * d code bytes and one
+    fp32 scale per row."""
+    codes, scale = sn.sn_quant_compress(X, fmt)
+    T, d = X.shape
+    return sn.sn_quant_restore(codes, scale, fmt), T * d + 4 * T
+
+
 def lowrank_roundtrip(X, r, power_iters=1, seed=0):
     T, d = X.shape
     gen = torch.Generator(device=X.device).manual_seed(seed)

@@ -541,6 +541,43 @@ sn_status sn_sign_restore(const uint32_t *bits, const float *scale, int64_t T, i
     return cuda_status(sn::lossy_sign_restore(bits, scale, T, d, X_out, (cudaStream_t)stream));
 }
 
+sn_status sn_quant_compress(const void *X, int64_t T, int32_t d, int32_t format, uint8_t *codes,
+                            float *scale, sn_stream_t stream)
+{
+    sn_status st = check_batch(X, T, d);
+    if (st != SN_OK)
+        return st;
+    if ((format != SN_Q_INT8 && format != SN_Q_E4M3) || !codes || !scale)
+        return SN_ERR_INVALID_ARG;
+    if (!aligned(codes, 8) || !aligned(scale, 4))
+        return SN_ERR_ALIGNMENT;
+    if (T == 0)
+        return SN_OK;
+    const size_t nx = (size_t)T * d * 2, nc = (size_t)T * d, ns = (size_t)T * 4;
+    if (overlap(X, nx, codes, nc) || overlap(X, nx, scale, ns) || overlap(codes, nc, scale, ns))
+        return SN_ERR_INVALID_ARG;
+    return cuda_status(sn::lossy_quant(X, T, d, format, codes, scale, (cudaStream_t)stream));
+}
+
+sn_status sn_quant_restore(const uint8_t *codes, const float *scale, int64_t T, int32_t d,
+                           int32_t format, void *X_out, sn_stream_t stream)
+{
+    sn_status st = check_batch(X_out, T, d);
+    if (st != SN_OK)
+        return st;
+    if ((format != SN_Q_INT8 && format != SN_Q_E4M3) || !codes || !scale)
+        return SN_ERR_INVALID_ARG;
+    if (!aligned(codes, 8) || !aligned(scale, 4))
+        return SN_ERR_ALIGNMENT;
+    if (T == 0)
+        return SN_OK;
+    const size_t nx = (size_t)T * d * 2;
+    if (overlap(X_out, nx, codes, (size_t)T * d) || overlap(X_out, nx, scale, (size_t)T * 4))
+        return SN_ERR_INVALID_ARG;
+    return cuda_status(sn::lossy_quant_restore(codes, scale, T, d, format, X_out,
+                                               (cudaStream_t)stream));
+}
+
 sn_status sn_wire_bytes(sn_basis_t b, sn_dtype dt, int64_t T, size_t *bytes)
 {
     if (!b || !bytes || T < 0 || (dt != SN_BF16 && dt != SN_F32))

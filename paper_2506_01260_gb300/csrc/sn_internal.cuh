@@ -102,6 +102,10 @@ cudaError_t lossy_sign(const void *X, int64_t T, int d, uint32_t *bits, float *s
                        cudaStream_t s);
 cudaError_t lossy_sign_restore(const uint32_t *bits, const float *scale, int64_t T, int d,
                                void *out, cudaStream_t s);
+cudaError_t lossy_quant(const void *X, int64_t T, int d, int format, uint8_t *codes, float *scale,
+                        cudaStream_t s);
+cudaError_t lossy_quant_restore(const uint8_t *codes, const float *scale, int64_t T, int d,
+                                int format, void *out, cudaStream_t s);
 // C = X U - TU[ids] - PU[pos] (PU may be null)
 cudaError_t tc_compress_projected(const sn_basis &b, const __nv_bfloat16 *X, const int32_t *ids,
                                   const int32_t *pos, int64_t T, int seq_len, const float *TU,

@@ -1,6 +1,7 @@
 // sn_lossy.cu — the lossy comparators of the paper's comparison at equal wire
-// size (Sec. 8, "Comparison against lossy compressions"): per-row top-k and
-// 1-bit sign quantization of a bf16 batch, with their restores.
+// size (Sec. 8, "Comparison against lossy compressions"): per-row top-k, 1-bit
+// sign quantization and row-scaled 8-bit quantization (int8, fp8 e4m3) of a
+// bf16 batch, with their restores.
 //
 // Top-k keeps the kk entries of largest magnitude of each row, ties towards the
 // lower column, and writes them in ascending column order.  One warp per row
@@ -23,6 +24,9 @@
 //           equal keys, kk > 128) the same search and placement run over the
 //           whole row, re-read from L2, skipping chunks whose maximum cannot
 //           matter.
+#include <cuda_fp16.h>
+#include <cuda_fp8.h>
+
 #include "sn_tc.cuh"
 
 namespace sn {
@@ -33,6 +37,7 @@ constexpr int kWarps = kThreads / 32;
 constexpr int kWCap = 256;                // candidate chunks and entries per warp
 constexpr int kLoadBatch = 8;             // 16-byte loads in flight per lane (top-k)
 constexpr int kSignUnroll = 8;            // 16-byte loads in flight per lane (sign)
+constexpr int kQuantUnroll = 8;           // 16-byte loads in flight per lane (8-bit)
 
 __device__ __forceinline__ uint32_t max_u16x2(uint32_t a, uint32_t b)
 {
@@ -390,6 +395,141 @@ __global__ void __launch_bounds__(kThreads) k_sign_restore(const uint32_t *__res
     }
 }
 
+// ---- Row-scaled 8-bit quantization -------------------------------------------
+// a = max |x| of the row, scale = a / qmax, code = Q(x * r) with r = qmax / a
+// (0 for a zero row): int8 rounds half to even and clamps to +-127, fp8 e4m3
+// rounds to nearest even and saturates at +-448.  The code is decided in fp32
+// from one rounded division per row and one rounded product per entry.
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+// the four codes of one packed word pair of bf16 (entries 0..3 in bytes 0..3)
+template <int FMT>
+__device__ __forceinline__ uint32_t quant4(uint32_t w0, uint32_t w1, float r)
+{
+    const float x0 = __fmul_rn(bf16_lo(w0), r), x1 = __fmul_rn(bf16_hi(w0), r);
+    const float x2 = __fmul_rn(bf16_lo(w1), r), x3 = __fmul_rn(bf16_hi(w1), r);
+    if (FMT == SN_Q_INT8) {
+        // |x| <= 127 (1 + 2^-23), so rint(x) already lies in [-127, 127].  Adding
+        // 1.5 * 2^23 rounds x to an integer (the fp32 addition rounds to nearest
+        // even at unit spacing) held in the low mantissa bits, whose low byte is
+        // rint(x) in two's complement; byte permutes gather the four low bytes.
+        constexpr float kRound = 12582912.0f;
+        const uint32_t q0 = __float_as_uint(__fadd_rn(x0, kRound));
+        const uint32_t q1 = __float_as_uint(__fadd_rn(x1, kRound));
+        const uint32_t q2 = __float_as_uint(__fadd_rn(x2, kRound));
+        const uint32_t q3 = __float_as_uint(__fadd_rn(x3, kRound));
+        return __byte_perm(__byte_perm(q0, q1, 0x0040), __byte_perm(q2, q3, 0x0040), 0x5410);
+    }
+    const uint32_t lo = __nv_cvt_float2_to_fp8x2(make_float2(x0, x1), __NV_SATFINITE, __NV_E4M3);
+    const uint32_t hi = __nv_cvt_float2_to_fp8x2(make_float2(x2, x3), __NV_SATFINITE, __NV_E4M3);
+    return lo | (hi << 16);
+}
+
+// One warp per row.  Pass 1 takes the largest magnitude from the low 15 bits
+// of every bf16 (they order the magnitudes of finite values); pass 2 reads
+// the row again (from L2) and writes each 16-byte chunk's 8 codes with one
+// 8-byte store, the warp's 32 stores one contiguous 256-byte run.
+template <int FMT>
+__global__ void __launch_bounds__(kThreads) k_quant(const uint16_t *__restrict__ X, int64_t T, int d,
+                                                     uint8_t *__restrict__ codes,
+                                                     float *__restrict__ scale)
+{
+    const int lane = threadIdx.x & 31;
+    const int64_t nwarps = ((int64_t)gridDim.x * kThreads) >> 5;
+    const int nch = d / 8;
+    const float qmax = FMT == SN_Q_INT8 ? 127.f : 448.f;
+    for (int64_t t = ((int64_t)blockIdx.x * kThreads + threadIdx.x) >> 5; t < T; t += nwarps) {
+        const uint4 *src = (const uint4 *)(X + t * (int64_t)d);
+        uint32_t m = 0;
+        for (int base = 0; base < nch; base += kQuantUnroll * 32) {
+            uint4 v[kQuantUnroll];
+#pragma unroll
+            for (int u = 0; u < kQuantUnroll; ++u) {
+                const int c = base + 32 * u + lane;
+                v[u] = c < nch ? __ldg(src + c) : make_uint4(0, 0, 0, 0);
+            }
+#pragma unroll
+            for (int u = 0; u < kQuantUnroll; ++u)
+                m = max_u16x2(m, max_u16x2(max_u16x2(v[u].x & 0x7FFF7FFFu, v[u].y & 0x7FFF7FFFu),
+                                           max_u16x2(v[u].z & 0x7FFF7FFFu, v[u].w & 0x7FFF7FFFu)));
+        }
+        m = __reduce_max_sync(0xffffffffu, max(m & 0xFFFFu, m >> 16));
+        const float a = __uint_as_float(m << 16);
+        const float r = a > 0.f ? qmax / a : 0.f;
+        uint2 *dst = (uint2 *)(codes + t * (int64_t)d);
+        for (int base = 0; base < nch; base += kQuantUnroll * 32) {
+            uint4 v[kQuantUnroll];
+#pragma unroll
+            for (int u = 0; u < kQuantUnroll; ++u) {
+                const int c = base + 32 * u + lane;
+                v[u] = c < nch ? __ldg(src + c) : make_uint4(0, 0, 0, 0);
+            }
+#pragma unroll
+            for (int u = 0; u < kQuantUnroll; ++u) {
+                const int c = base + 32 * u + lane;
+                if (c < nch)
+                    dst[c] = make_uint2(quant4<FMT>(v[u].x, v[u].y, r), quant4<FMT>(v[u].z, v[u].w, r));
+            }
+        }
+        if (lane == 0)
+            scale[t] = a / qmax;
+    }
+}
+
+// the values of four codes (bytes 0..3 of q)
+template <int FMT>
+__device__ __forceinline__ void dequant4(uint32_t q, float (&f)[4])
+{
+    if (FMT == SN_Q_INT8) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+            f[e] = (float)(int8_t)(q >> (8 * e));
+        return;
+    }
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const __half2_raw raw =
+            __nv_cvt_fp8x2_to_halfraw2((__nv_fp8x2_storage_t)(q >> (16 * h)), __NV_E4M3);
+        const float2 v = __half22float2(__half2(raw));
+        f[2 * h] = v.x;
+        f[2 * h + 1] = v.y;
+    }
+}
+
+__device__ __forceinline__ uint32_t bf16x2_rn(float lo, float hi)
+{
+    const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *(const uint32_t *)&v;
+}
+
+// Restore: one warp per row; per lane 8 codes in, decode(code) * scale in
+// fp32, one rounding to bf16, one 16-byte store.
+template <int FMT>
+__global__ void __launch_bounds__(kThreads) k_quant_restore(const uint8_t *__restrict__ codes,
+                                                             const float *__restrict__ scale,
+                                                             int64_t T, int d,
+                                                             uint16_t *__restrict__ out)
+{
+    const int lane = threadIdx.x & 31;
+    const int64_t nwarps = ((int64_t)gridDim.x * kThreads) >> 5;
+    const int nch = d / 8;
+    for (int64_t t = ((int64_t)blockIdx.x * kThreads + threadIdx.x) >> 5; t < T; t += nwarps) {
+        const float s = scale[t];
+        const uint2 *src = (const uint2 *)(codes + t * (int64_t)d);
+        uint4 *dst = (uint4 *)(out + t * (int64_t)d);
+        for (int c = lane; c < nch; c += 32) {
+            const uint2 q = __ldg(src + c);
+            float f[8];
+            dequant4<FMT>(q.x, *(float(*)[4])f);
+            dequant4<FMT>(q.y, *(float(*)[4])(f + 4));
+            dst[c] = make_uint4(bf16x2_rn(f[0] * s, f[1] * s), bf16x2_rn(f[2] * s, f[3] * s),
+                                bf16x2_rn(f[4] * s, f[5] * s), bf16x2_rn(f[6] * s, f[7] * s));
+        }
+    }
+}
+
 int row_grid(int64_t T)
 {
     int dev = 0, sms = 148;
@@ -461,6 +601,46 @@ cudaError_t lossy_sign(const void *X, int64_t T, int d, uint32_t *bits, float *s
                        cudaStream_t s)
 {
     k_sign<<<warp_grid(T), kThreads, 0, s>>>((const uint16_t *)X, T, d, bits, scale);
+    count_launch();
+    return cudaGetLastError();
+}
+
+// The 8-bit quantizer reads every row twice; the second read hits L2 only if
+// the rows in flight (one per warp) stay well inside it, so the grid keeps
+// them under 48 MiB: 2 CTAs of 8 warps per SM at d = 8192, up to 8 for short
+// rows.
+int quant_grid(int64_t T, int d)
+{
+    int dev = 0, sms = 148;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int64_t per_sm = ((int64_t)48 << 20) / ((int64_t)sms * kWarps * 2 * d);
+    const int64_t ctas = (per_sm < 1 ? 1 : per_sm > 8 ? 8 : per_sm) * sms;
+    const int64_t need = (T + kWarps - 1) / kWarps;
+    return (int)(need < ctas ? need : ctas);
+}
+
+cudaError_t lossy_quant(const void *X, int64_t T, int d, int format, uint8_t *codes, float *scale,
+                        cudaStream_t s)
+{
+    const int grid = quant_grid(T, d);
+    if (format == SN_Q_INT8)
+        k_quant<SN_Q_INT8><<<grid, kThreads, 0, s>>>((const uint16_t *)X, T, d, codes, scale);
+    else
+        k_quant<SN_Q_E4M3><<<grid, kThreads, 0, s>>>((const uint16_t *)X, T, d, codes, scale);
+    count_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t lossy_quant_restore(const uint8_t *codes, const float *scale, int64_t T, int d,
+                                int format, void *out, cudaStream_t s)
+{
+    if (format == SN_Q_INT8)
+        k_quant_restore<SN_Q_INT8><<<warp_grid(T), kThreads, 0, s>>>(codes, scale, T, d,
+                                                                     (uint16_t *)out);
+    else
+        k_quant_restore<SN_Q_E4M3><<<warp_grid(T), kThreads, 0, s>>>(codes, scale, T, d,
+                                                                     (uint16_t *)out);
     count_launch();
     return cudaGetLastError();
 }

@@ -59,6 +59,8 @@ _sig("sn_topk_compress", [_P, _I64, _I32, _I32, _P, _P, _P])
 _sig("sn_topk_restore", [_P, _P, _I64, _I32, _I32, _P, _P])
 _sig("sn_sign_compress", [_P, _I64, _I32, _P, _P, _P])
 _sig("sn_sign_restore", [_P, _P, _I64, _I32, _P, _P])
+_sig("sn_quant_compress", [_P, _I64, _I32, _I32, _P, _P, _P])
+_sig("sn_quant_restore", [_P, _P, _I64, _I32, _I32, _P, _P])
 _sig("sn_wire_bytes", [_P, _ST, _I64, ctypes.POINTER(_SZ)])
 _sig("sn_wire_send", [_P, _P, _SZ, _P])
 _sig("sn_wire_recv", [_P, _P, _SZ, _P])
@@ -74,7 +76,7 @@ EXPORTS = ["sn_basis_create", "sn_basis_destroy", "sn_basis_shape", "sn_compress
            "sn_project_tables", "sn_compress_fwd_projected", "sn_build_ts",
            "sn_grassmann_workspace", "sn_grassmann_accumulate", "sn_grassmann_residual",
            "sn_grassmann_step", "sn_adamw_rowconst", "sn_topk_compress", "sn_topk_restore",
-           "sn_sign_compress", "sn_sign_restore",
+           "sn_sign_compress", "sn_sign_restore", "sn_quant_compress", "sn_quant_restore",
            "sn_wire_bytes", "sn_wire_send",
            "sn_wire_recv", "sn_check_errors", "sn_selftest_wait_timeout", "sn_launch_count",
            "sn_status_string"]
@@ -380,6 +382,39 @@ def sn_sign_restore(bits, scale, d, out=None, stream=None):
         out = torch.empty(T, d, dtype=torch.bfloat16, device=scale.device)
     _check(_lib.sn_sign_restore(_ptr(bits), _ptr(scale), T, d, _ptr(out), _stream(stream)),
            "sn_sign_restore")
+    return out
+
+
+#: 8-bit formats of sn_quant_compress
+QUANT_FORMATS = {"int8": 0, "e4m3": 1}
+
+
+def sn_quant_compress(X, fmt, codes=None, scale=None, stream=None):
+    """Row-scaled 8-bit codes (uint8 [T, d]) and fp32 row scales max|x| / qmax [T];
+    fmt "int8" (qmax 127) or "e4m3" (fp8, qmax 448)."""
+    _need(X, "X", torch.bfloat16)
+    T, d = X.shape
+    if codes is None:
+        codes = torch.empty(T, d, dtype=torch.uint8, device=X.device)
+    if scale is None:
+        scale = torch.empty(T, dtype=torch.float32, device=X.device)
+    _need(codes, "codes", torch.uint8)
+    _need(scale, "scale", torch.float32)
+    if codes.shape != (T, d) or scale.shape != (T,):
+        raise ValueError("codes must be [T, d] and scale [T]")
+    _check(_lib.sn_quant_compress(_ptr(X), T, d, QUANT_FORMATS[fmt], _ptr(codes), _ptr(scale),
+                                  _stream(stream)), "sn_quant_compress")
+    return codes, scale
+
+
+def sn_quant_restore(codes, scale, fmt, out=None, stream=None):
+    _need(codes, "codes", torch.uint8)
+    _need(scale, "scale", torch.float32)
+    T, d = codes.shape
+    if out is None:
+        out = torch.empty(T, d, dtype=torch.bfloat16, device=codes.device)
+    _check(_lib.sn_quant_restore(_ptr(codes), _ptr(scale), T, d, QUANT_FORMATS[fmt], _ptr(out),
+                                 _stream(stream)), "sn_quant_restore")
     return out
 
 

@@ -1,7 +1,7 @@
 """GPU parity of the lossy comparators against the fp64 oracle in
 oracle/lossy.py: top-k columns, values and restores bit-exact (selection on bf16
 magnitudes, ties towards the lower column); sign bits exact and the row scale
-within 1e-6 relative; the randomized low-rank round trip within 1.5 times the
+within 1e-6 relative; int8 and fp8 e4m3 codes, scales and restores bit-exact; the randomized low-rank round trip within 1.5 times the
 error of the exact truncated SVD (plus 1e-3) on a noisy low-rank batch."""
 import importlib.util
 import os
@@ -98,3 +98,43 @@ def test_lossy_argument_errors(sn):
     with pytest.raises(sn.SNError) as e:
         sn.sn_sign_compress(torch.zeros(4, 60, dtype=torch.bfloat16, device="cuda"))   # d % 8
     assert e.value.status == sn.SN_ERR_INVALID_ARG
+
+
+# Row-scaled 8-bit quantization: codes, scales and restores bit for bit against
+# the oracle's fp32 decisions.  Rows of mixed magnitudes (2^-8 .. 2^8), a zero
+# row, a row with one nonzero entry, signed zeros and entries small enough to
+# round to (signed) zero in e4m3.
+@pytest.mark.parametrize("fmt", ["int8", "e4m3"])
+@pytest.mark.parametrize("T,d", [(1, 8), (37, 264), (300, 4096), (4, 65536), (9, 8200)])
+def test_quant_bit_exact(sn, fmt, T, d):
+    o = lossy_oracle()
+    rng = np.random.default_rng(3 * T + d)
+    x = rng.standard_normal((T, d)) * np.exp2(rng.uniform(-8, 8, (T, 1)))
+    x[0, :4] = [-0.0, 0.0, 1e-7 * np.abs(x[0]).max(), -1e-7 * np.abs(x[0]).max()]
+    if T >= 3:
+        x[1] = 0.0
+        x[2] = 0.0
+        x[2, d // 2] = -3.0
+    xb = W.to_bf16(x)
+    codes, scale = sn.sn_quant_compress(dev(xb), fmt)
+    rc, rs = o.quant_compress(xb, fmt)
+    assert np.array_equal(host(codes), rc)
+    assert np.array_equal(host(scale).view(np.uint32), rs.view(np.uint32))
+    back = sn.sn_quant_restore(codes, scale, fmt)
+    assert np.array_equal(host(back), o.quant_restore(rc, rs, fmt))
+
+
+def test_quant_argument_errors(sn):
+    X = torch.zeros(4, 64, dtype=torch.bfloat16, device="cuda")
+    codes = torch.empty(4, 64, dtype=torch.uint8, device="cuda")
+    scale = torch.empty(4, dtype=torch.float32, device="cuda")
+    lib = sn._lib
+    st = lib.sn_quant_compress(X.data_ptr(), 4, 64, 2, codes.data_ptr(), scale.data_ptr(), None)
+    assert st == sn.SN_ERR_INVALID_ARG                  # unknown format
+    st = lib.sn_quant_compress(X.data_ptr(), 4, 64, 0, codes.data_ptr() + 4, scale.data_ptr(),
+                               None)
+    assert st == sn.SN_ERR_ALIGNMENT                    # codes not 8-byte aligned
+    st = lib.sn_quant_restore(codes.data_ptr(), scale.data_ptr(), 4, 60, 1, X.data_ptr(), None)
+    assert st == sn.SN_ERR_INVALID_ARG                  # d % 8
+    st = lib.sn_quant_compress(X.data_ptr(), 4, 64, 1, X.data_ptr(), scale.data_ptr(), None)
+    assert st == sn.SN_ERR_INVALID_ARG                  # codes overlap X

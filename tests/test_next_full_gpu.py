@@ -7,9 +7,9 @@ calls the benchmark times, on samples the fp64 oracles compute one by one:
   time;
 - the row-constant AdamW step on W_o [8192, 8192] (Sec. 5): sampled columns
   (each column's rate depends only on that column);
-- the top-k and sign comparators on X (Sec. 8): sampled rows.
+- the top-k, sign and 8-bit comparators on X (Sec. 8): sampled rows.
 Bars as everywhere: 1e-2 relative Frobenius error for bf16 results, 1e-5 for
-fp32 ones, exact for selected columns and sign bits."""
+fp32 ones, exact for selected columns, sign bits and 8-bit codes."""
 import importlib.util
 import os
 
@@ -129,3 +129,8 @@ def test_lossy_comparators_full_size(sn, large):
     got = ((words[:, :, None] >> np.arange(32)[None, None, :]) & 1).reshape(len(rows), -1)
     assert np.array_equal(got[:, :wl.d].astype(np.uint8), rb)
     assert np.max(np.abs(host(scale[rt]).astype(np.float64) - rs) / rs) <= 1e-6
+    for fmt in ("int8", "e4m3"):
+        codes, qs = sn.sn_quant_compress(X, fmt)
+        rc, rq = o.quant_compress(xb, fmt)
+        assert np.array_equal(host(codes[rt]), rc), fmt
+        assert np.array_equal(host(qs[rt]).view(np.uint32), rq.view(np.uint32)), fmt
