@@ -263,8 +263,9 @@ sn_status sn_sign_compress(const void *X, int64_t T, int32_t d, uint32_t *bits, 
 sn_status sn_sign_restore(const uint32_t *bits, const float *scale, int64_t T, int32_t d,
                           void *X_out, sn_stream_t stream);
 
-/* Row-scaled 8-bit quantization, the comparison's quantizer at twice the
- * rate of the 1-bit one's bits per entry (X finite).  Per row t:
+/* Row-scaled 8-bit quantization (int8 or fp8 e4m3): rate points of the
+ * comparison's quantizer beside the 1-bit one.  X finite; a row whose largest
+ * magnitude lies in (0, 2^-119) is outside the domain.  Per row t:
  * a = max |X[t, :]|, scale[t] = a / qmax (fp32), codes[t, c] = Q(X[t, c] * r)
  * with r = qmax / a (0 for a zero row), both fp32 operations.
  *   SN_Q_INT8  qmax = 127, Q = round half to even, clamp to [-127, 127],
