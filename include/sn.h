@@ -11,9 +11,11 @@
  * S by projecting them with P = U U^T (Sec. 4.3, Sec. 5, App. A).
  *
  * Conventions shared by every call
- *   - Tensor pointers are device pointers (memory of the current CUDA device)
- *     unless stated otherwise, owned by the caller, contiguous row-major, and
- *     16-byte aligned (SN_ERR_ALIGNMENT otherwise).
+ *   - Tensor pointers are device pointers (memory of the current CUDA device,
+ *     or managed memory) unless stated otherwise, owned by the caller,
+ *     contiguous row-major, and 16-byte aligned (SN_ERR_ALIGNMENT otherwise).
+ *     Host memory, pageable or pinned, is refused with SN_ERR_INVALID_ARG
+ *     (checked with cudaPointerGetAttributes) rather than handed to a kernel.
  *   - Calls are stream-ordered and asynchronous: they validate their
  *     arguments, enqueue kernels on `stream` and return.  An argument error
  *     returns synchronously and enqueues nothing.

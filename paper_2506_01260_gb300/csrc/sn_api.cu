@@ -3,6 +3,7 @@
 // CUDA-core kernels), the wire copies and the asynchronous error word.
 #include <atomic>
 #include <cstdlib>
+#include <initializer_list>
 #include <new>
 
 #include "sn_internal.cuh"
@@ -28,6 +29,31 @@ bool overlap(const void *a, size_t na, const void *b, size_t nb)
 size_t esize(sn_dtype dt) { return dt == SN_BF16 ? 2 : 4; }
 
 sn_status cuda_status(cudaError_t e) { return e == cudaSuccess ? SN_OK : SN_ERR_CUDA; }
+
+// Kernels dereference every tensor pointer, so each must be device memory of
+// the current device or managed memory; host memory (pageable or pinned) is
+// refused here instead of faulting in a kernel.  Null pointers are left to the
+// callers' own checks.
+bool on_device(std::initializer_list<const void *> ptrs)
+{
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess)
+        return false;
+    for (const void *p : ptrs) {
+        if (!p)
+            continue;
+        cudaPointerAttributes a;
+        if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+            (void)cudaGetLastError();
+            return false;
+        }
+        if (a.type == cudaMemoryTypeManaged)
+            continue;
+        if (a.type != cudaMemoryTypeDevice || a.device != dev)
+            return false;
+    }
+    return true;
+}
 
 // Common checks of a basis handle and dtype; the handle must live on the
 // current device.
@@ -62,7 +88,7 @@ sn_status check_fwd(sn_basis_t b, sn_dtype dt, const void *in, const int32_t *id
     const size_t es = esize(dt);
     if (overlap(in, (size_t)T * in_row * es, out, (size_t)T * out_row * es))
         return SN_ERR_INVALID_ARG;
-    return SN_OK;
+    return on_device({in, ids, pos, tok, pe, out}) ? SN_OK : SN_ERR_INVALID_ARG;
 }
 
 }  // namespace
@@ -93,6 +119,8 @@ sn_status sn_basis_create(const float *U, int32_t d, int32_t k, sn_basis_t *out,
         return SN_ERR_INVALID_ARG;
     if (!aligned(U, 16))
         return SN_ERR_ALIGNMENT;
+    if (!on_device({U}))
+        return SN_ERR_INVALID_ARG;
     sn_basis *b = new (std::nothrow) sn_basis();
     if (!b)
         return SN_ERR_CUDA;
@@ -201,7 +229,7 @@ sn_status sn_compress_bwd(sn_basis_t b, sn_dtype dt, const void *G, int64_t T, v
     if (!aligned(G, 16) || !aligned(C, 16))
         return SN_ERR_ALIGNMENT;
     const size_t es = esize(dt);
-    if (overlap(G, (size_t)T * b->d * es, C, (size_t)T * b->k * es))
+    if (overlap(G, (size_t)T * b->d * es, C, (size_t)T * b->k * es) || !on_device({G, C}))
         return SN_ERR_INVALID_ARG;
     cudaStream_t s = (cudaStream_t)stream;
     if (dt == SN_F32)
@@ -227,7 +255,7 @@ sn_status sn_decompress_bwd(sn_basis_t b, sn_dtype dt, const void *C, int64_t T,
     if (!aligned(G, 16) || !aligned(C, 16))
         return SN_ERR_ALIGNMENT;
     const size_t es = esize(dt);
-    if (overlap(G, (size_t)T * b->d * es, C, (size_t)T * b->k * es))
+    if (overlap(G, (size_t)T * b->d * es, C, (size_t)T * b->k * es) || !on_device({G, C}))
         return SN_ERR_INVALID_ARG;
     cudaStream_t s = (cudaStream_t)stream;
     if (dt == SN_F32)
@@ -277,7 +305,8 @@ sn_status sn_project_weight(sn_basis_t b, sn_dtype dt, const void *W, int64_t ro
     const size_t wbytes = ((size_t)(rows - 1) * ld + cols) * es;
     if (W != W_out && overlap(W, wbytes, W_out, wbytes))
         return SN_ERR_INVALID_ARG;
-    if (overlap(ws, need, W, wbytes) || overlap(ws, need, W_out, wbytes))
+    if (overlap(ws, need, W, wbytes) || overlap(ws, need, W_out, wbytes) ||
+        !on_device({W, W_out, ws}))
         return SN_ERR_INVALID_ARG;
     cudaStream_t s = (cudaStream_t)stream;
     if (dt == SN_F32)
@@ -303,7 +332,8 @@ sn_status sn_project_tables(sn_basis_t b, sn_dtype dt, const void *tok, int64_t 
         return SN_ERR_ALIGNMENT;
     if (overlap(tok, (size_t)vocab * b->d * 2, TU, (size_t)vocab * b->k * 4) ||
         (pe && (overlap(pe, (size_t)seq_len * b->d * 2, PU, (size_t)seq_len * b->k * 4) ||
-                overlap(TU, (size_t)vocab * b->k * 4, PU, (size_t)seq_len * b->k * 4))))
+                overlap(TU, (size_t)vocab * b->k * 4, PU, (size_t)seq_len * b->k * 4))) ||
+        !on_device({tok, pe, TU, PU}))
         return SN_ERR_INVALID_ARG;
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t e = sn::tc_contract_f32(*b, (const __nv_bfloat16 *)tok, vocab, TU, s);
@@ -344,7 +374,7 @@ sn_status sn_build_ts(sn_basis_t b, sn_dtype dt, const void *tok, int64_t vocab,
     if (!aligned(tok, 16) || !aligned(T_S, 16) || !aligned(ws, 16))
         return SN_ERR_ALIGNMENT;
     if (overlap(tok, table, T_S, table) || overlap(tok, table, ws, coeff) ||
-        overlap(T_S, table, ws, coeff))
+        overlap(T_S, table, ws, coeff) || !on_device({tok, T_S, ws}))
         return SN_ERR_INVALID_ARG;
     cudaStream_t s = (cudaStream_t)stream;
     sn::TcArgs a{(const __nv_bfloat16 *)tok, nullptr, nullptr, nullptr, nullptr,
@@ -389,7 +419,7 @@ sn_status sn_grassmann_accumulate(sn_basis_t b, sn_dtype dt, const void *G, cons
     const size_t mb = (size_t)b->d * b->k * 4;
     if (overlap(M, mb, G, (size_t)T * b->d * 2) || overlap(M, mb, Cg, (size_t)T * b->k * 2) ||
         overlap(ws, ws_bytes, M, mb) || overlap(ws, ws_bytes, G, (size_t)T * b->d * 2) ||
-        overlap(ws, ws_bytes, Cg, (size_t)T * b->k * 2))
+        overlap(ws, ws_bytes, Cg, (size_t)T * b->k * 2) || !on_device({G, Cg, M, ws}))
         return SN_ERR_INVALID_ARG;
     return cuda_status(sn::tc_grassmann_accumulate(*b, (const __nv_bfloat16 *)G,
                                                    (const __nv_bfloat16 *)Cg, T, M, ws,
@@ -412,6 +442,8 @@ sn_status sn_grassmann_residual(sn_basis_t b, sn_dtype dt, const void *G, const 
         return SN_ERR_INVALID_ARG;
     if (!aligned(G, 16) || !aligned(Cg, 2) || !aligned(acc, 8))
         return SN_ERR_ALIGNMENT;
+    if (!on_device({G, Cg, acc}))
+        return SN_ERR_INVALID_ARG;
     return cuda_status(sn::grassmann_residual(*b, (const __nv_bfloat16 *)G,
                                               (const __nv_bfloat16 *)Cg, T, acc,
                                               (cudaStream_t)stream));
@@ -430,7 +462,7 @@ sn_status sn_grassmann_step(sn_basis_t b, const float *M, int32_t K, float eta, 
         return SN_ERR_ALIGNMENT;
     const size_t mb = (size_t)b->d * b->k * 4;
     if (overlap(M, mb, U_new, mb) || overlap(ws, ws_bytes, M, mb) ||
-        overlap(ws, ws_bytes, U_new, mb))
+        overlap(ws, ws_bytes, U_new, mb) || !on_device({M, U_new, ws}))
         return SN_ERR_INVALID_ARG;
     return cuda_status(sn::grassmann_step(*b, M, K, eta, U_new, ws, (cudaStream_t)stream));
 }
@@ -455,6 +487,8 @@ sn_status sn_adamw_rowconst(sn_dtype gdt, float *W, const void *g, float *M, flo
         for (int j = i + 1; j < 5; ++j)
             if (overlap(bufs[i], lens[i], bufs[j], lens[j]))
                 return SN_ERR_INVALID_ARG;
+    if (!on_device({W, g, M, V, ws}))
+        return SN_ERR_INVALID_ARG;
     return cuda_status(sn::adamw_rowconst(gdt == SN_BF16, W, g, M, V, rows, cols, t, lr, b1, b2,
                                           eps, lam, (float *)ws, (cudaStream_t)stream));
 }
@@ -481,7 +515,8 @@ sn_status sn_topk_compress(const void *X, int64_t T, int32_t d, int32_t kk, void
     if (T == 0)
         return SN_OK;
     const size_t nx = (size_t)T * d * 2, nk = (size_t)T * kk * 2;
-    if (overlap(X, nx, vals, nk) || overlap(X, nx, cols, nk) || overlap(vals, nk, cols, nk))
+    if (overlap(X, nx, vals, nk) || overlap(X, nx, cols, nk) || overlap(vals, nk, cols, nk) ||
+        !on_device({X, vals, cols}))
         return SN_ERR_INVALID_ARG;
     return cuda_status(sn::lossy_topk(X, T, d, kk, vals, cols, (cudaStream_t)stream));
 }
@@ -499,7 +534,8 @@ sn_status sn_topk_restore(const void *vals, const uint16_t *cols, int64_t T, int
     if (T == 0)
         return SN_OK;
     const size_t nx = (size_t)T * d * 2, nk = (size_t)T * kk * 2;
-    if (overlap(X_out, nx, vals, nk) || overlap(X_out, nx, cols, nk))
+    if (overlap(X_out, nx, vals, nk) || overlap(X_out, nx, cols, nk) ||
+        !on_device({vals, cols, X_out}))
         return SN_ERR_INVALID_ARG;
     return cuda_status(sn::lossy_topk_restore(vals, cols, T, d, kk, X_out, (cudaStream_t)stream));
 }
@@ -517,7 +553,8 @@ sn_status sn_sign_compress(const void *X, int64_t T, int32_t d, uint32_t *bits, 
     if (T == 0)
         return SN_OK;
     const size_t nx = (size_t)T * d * 2, nb = (size_t)T * ((d + 31) / 32) * 4, ns = (size_t)T * 4;
-    if (overlap(X, nx, bits, nb) || overlap(X, nx, scale, ns) || overlap(bits, nb, scale, ns))
+    if (overlap(X, nx, bits, nb) || overlap(X, nx, scale, ns) || overlap(bits, nb, scale, ns) ||
+        !on_device({X, bits, scale}))
         return SN_ERR_INVALID_ARG;
     return cuda_status(sn::lossy_sign(X, T, d, bits, scale, (cudaStream_t)stream));
 }
@@ -536,7 +573,7 @@ sn_status sn_sign_restore(const uint32_t *bits, const float *scale, int64_t T, i
         return SN_OK;
     const size_t nx = (size_t)T * d * 2;
     if (overlap(X_out, nx, bits, (size_t)T * ((d + 31) / 32) * 4) ||
-        overlap(X_out, nx, scale, (size_t)T * 4))
+        overlap(X_out, nx, scale, (size_t)T * 4) || !on_device({bits, scale, X_out}))
         return SN_ERR_INVALID_ARG;
     return cuda_status(sn::lossy_sign_restore(bits, scale, T, d, X_out, (cudaStream_t)stream));
 }
@@ -554,7 +591,8 @@ sn_status sn_quant_compress(const void *X, int64_t T, int32_t d, int32_t format,
     if (T == 0)
         return SN_OK;
     const size_t nx = (size_t)T * d * 2, nc = (size_t)T * d, ns = (size_t)T * 4;
-    if (overlap(X, nx, codes, nc) || overlap(X, nx, scale, ns) || overlap(codes, nc, scale, ns))
+    if (overlap(X, nx, codes, nc) || overlap(X, nx, scale, ns) || overlap(codes, nc, scale, ns) ||
+        !on_device({X, codes, scale}))
         return SN_ERR_INVALID_ARG;
     return cuda_status(sn::lossy_quant(X, T, d, format, codes, scale, (cudaStream_t)stream));
 }
@@ -572,7 +610,8 @@ sn_status sn_quant_restore(const uint8_t *codes, const float *scale, int64_t T, 
     if (T == 0)
         return SN_OK;
     const size_t nx = (size_t)T * d * 2;
-    if (overlap(X_out, nx, codes, (size_t)T * d) || overlap(X_out, nx, scale, (size_t)T * 4))
+    if (overlap(X_out, nx, codes, (size_t)T * d) || overlap(X_out, nx, scale, (size_t)T * 4) ||
+        !on_device({codes, scale, X_out}))
         return SN_ERR_INVALID_ARG;
     return cuda_status(sn::lossy_quant_restore(codes, scale, T, d, format, X_out,
                                                (cudaStream_t)stream));
@@ -590,7 +629,7 @@ sn_status sn_wire_send(const void *src_device, void *dst_host, size_t bytes, sn_
 {
     if (bytes == 0)
         return SN_OK;
-    if (!src_device || !dst_host)
+    if (!src_device || !dst_host || !on_device({src_device}))
         return SN_ERR_INVALID_ARG;
     return cuda_status(cudaMemcpyAsync(dst_host, src_device, bytes, cudaMemcpyDeviceToHost,
                                        (cudaStream_t)stream));
@@ -600,7 +639,7 @@ sn_status sn_wire_recv(const void *src_host, void *dst_device, size_t bytes, sn_
 {
     if (bytes == 0)
         return SN_OK;
-    if (!src_host || !dst_device)
+    if (!src_host || !dst_device || !on_device({dst_device}))
         return SN_ERR_INVALID_ARG;
     return cuda_status(cudaMemcpyAsync(dst_device, src_host, bytes, cudaMemcpyHostToDevice,
                                        (cudaStream_t)stream));

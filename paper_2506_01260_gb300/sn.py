@@ -115,6 +115,8 @@ def _ptr(t):
 def _need(t, name, dtype=None, contiguous=True):
     if not isinstance(t, torch.Tensor):
         raise TypeError("%s must be a torch.Tensor" % name)
+    if not t.is_cuda:
+        raise ValueError("%s must be a CUDA tensor" % name)
     if dtype is not None and t.dtype != dtype:
         raise TypeError("%s must be %s, got %s" % (name, dtype, t.dtype))
     if contiguous and not t.is_contiguous():
@@ -524,6 +526,8 @@ def sn_wire_bytes(basis, dtype, T):
 def sn_wire_send(src_device, dst_host, stream=None):
     """Device tensor -> (pinned) host tensor of the same byte size."""
     n = src_device.numel() * src_device.element_size()
+    if not src_device.is_cuda:
+        raise ValueError("source must be a CUDA tensor")
     if dst_host.numel() * dst_host.element_size() < n or dst_host.is_cuda:
         raise ValueError("destination must be host memory of at least %d bytes" % n)
     _check(_lib.sn_wire_send(_ptr(src_device), _ptr(dst_host), n, _stream(stream)),
@@ -534,6 +538,8 @@ def sn_wire_send(src_device, dst_host, stream=None):
 def sn_wire_recv(src_host, dst_device, stream=None):
     """(Pinned) host tensor -> device tensor of the same byte size."""
     n = src_host.numel() * src_host.element_size()
+    if src_host.is_cuda:
+        raise ValueError("source must be host memory")
     if dst_device.numel() * dst_device.element_size() < n or not dst_device.is_cuda:
         raise ValueError("destination must be device memory of at least %d bytes" % n)
     _check(_lib.sn_wire_recv(_ptr(src_host), _ptr(dst_device), n, _stream(stream)),

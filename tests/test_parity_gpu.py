@@ -6,6 +6,8 @@ counts and layouts.  Sizes span several 128-token tiles with ragged tails, k
 from 1 to 128, d from 16 to 8192; guard bands around every output catch
 out-of-bounds writes.
 """
+import ctypes
+
 import numpy as np
 import pytest
 import torch
@@ -414,4 +416,51 @@ def test_split_last_round(sn, oracle, layout):
         _, C64, _ = oracle.compress_fwd(inp["X"], inp["ids"], inp["tok_emb"], inp["U"], n,
                                         pos_emb=inp["pos_emb"], pos=pos)
         assert rel_fro(host(C), C64) <= TOL["bf16"]
+    basis.destroy()
+
+
+def test_host_pointers_are_refused(sn):
+    """Every tensor argument must be device memory of the current device: host
+    memory (pageable or pinned) is refused with SN_ERR_INVALID_ARG before any
+    launch, in the binding and at the C ABI."""
+    T, d, k, n, vocab = 256, 256, 8, 128, 1024
+    U = torch.linalg.qr(torch.randn(d, k, dtype=torch.float64))[0].float().contiguous().cuda()
+    basis = sn.Basis(U)
+    with pytest.raises(ValueError):
+        sn.Basis(U.cpu())
+    st = sn._lib.sn_basis_create(ctypes.c_void_p(U.cpu().data_ptr()), d, k,
+                                 ctypes.byref(ctypes.c_void_p()), None)
+    assert st == sn.SN_ERR_INVALID_ARG
+    X = torch.zeros(T, d, dtype=torch.bfloat16, device="cuda")
+    ids = torch.zeros(T, dtype=torch.int32, device="cuda")
+    tok = torch.zeros(vocab, d, dtype=torch.bfloat16, device="cuda")
+    C = torch.empty(T, k, dtype=torch.bfloat16, device="cuda")
+    launches = sn.sn_launch_count()
+    with pytest.raises(ValueError):
+        sn.sn_compress_fwd(basis, X.cpu(), ids, tok, n, out=C)
+    lib, P = sn._lib, ctypes.c_void_p
+    for host in (X.cpu(), X.cpu().pin_memory()):
+        st = lib.sn_compress_fwd(basis.handle, sn.SN_BF16, P(host.data_ptr()), P(ids.data_ptr()),
+                                 None, T, n, P(tok.data_ptr()), vocab, None, P(C.data_ptr()),
+                                 None)
+        assert st == sn.SN_ERR_INVALID_ARG
+        st = lib.sn_decompress_fwd(basis.handle, sn.SN_BF16, P(C.data_ptr()), P(ids.data_ptr()),
+                                   None, T, n, P(tok.data_ptr()), vocab, None,
+                                   P(host.data_ptr()), None)
+        assert st == sn.SN_ERR_INVALID_ARG
+        st = lib.sn_compress_bwd(basis.handle, sn.SN_BF16, P(host.data_ptr()), T,
+                                 P(C.data_ptr()), None)
+        assert st == sn.SN_ERR_INVALID_ARG
+        codes = torch.empty(T, d, dtype=torch.uint8, device="cuda")
+        scale = torch.empty(T, dtype=torch.float32, device="cuda")
+        st = lib.sn_quant_compress(P(host.data_ptr()), T, d, 0, P(codes.data_ptr()),
+                                   P(scale.data_ptr()), None)
+        assert st == sn.SN_ERR_INVALID_ARG
+    ids_host = ids.cpu()
+    st = lib.sn_compress_fwd(basis.handle, sn.SN_BF16, P(X.data_ptr()), P(ids_host.data_ptr()),
+                             None, T, n, P(tok.data_ptr()), vocab, None, P(C.data_ptr()), None)
+    assert st == sn.SN_ERR_INVALID_ARG
+    assert sn.sn_launch_count() == launches        # nothing was launched
+    sn.sn_compress_fwd(basis, X, ids, tok, n, out=C)  # device memory still works
+    sn.sn_check_errors(basis)
     basis.destroy()
