@@ -3,7 +3,8 @@
 Bar (relative Frobenius error against the oracle's unrounded fp64 value):
 1e-2 for bf16 outputs, 1e-5 for fp32 outputs; bit-exact for gathers, wire byte
 counts and layouts.  Sizes span several 128-token tiles with ragged tails, k
-from 1 to 128, d from 16 to 8192; guard bands around every output catch
+from 1 to 128, d from 16 to 16384 (including widths that end in a partial
+64-column chunk and 128-column block); guard bands around every output catch
 out-of-bounds writes.
 """
 import ctypes
@@ -27,6 +28,10 @@ CASES = [
     ("one_token_d64_k1", 1, 7, 64, 1, 5),
     ("square_d16_k16", 70, 9, 16, 16, 33),
     ("exact_tile_d256_k16", 256, 128, 256, 16, 300),
+    ("ragged_chunk_d200_k24", 300, 50, 200, 24, 700),      # d: 3 chunks of 64 + 8; blocks 128 + 72
+    ("ragged_chunk_d2056_k33", 257, 64, 2056, 33, 900),
+    ("wide_d12288_k96", 150, 64, 12288, 96, 400),
+    ("wide_d16384_k128", 131, 32, 16384, 128, 300),
 ]
 DTYPES = ["bf16", "f32"]
 
