@@ -369,6 +369,28 @@ def lossy_comparison(args, sn, basis, X, Xr, ids, tok, pe, n, flush, stream, hbm
     return out
 
 
+def paper_context(T, d, k, codec_ms, link_mbps=80.0):
+    """The paper's own figures (other hardware, other setting), reported beside
+    the measurement as context, not as its target: the compression ratio of the
+    wire against the activation (Sec. 1, Sec. 8.1: up to 99%, ~100x at k = 40,
+    d = 4096) and what one step's boundary traffic costs on the consumer links
+    of its experiments (80 Mbps, Sec. 8.1) with and without the codec."""
+    wire = 2 * (T * k * 2)                   # C forward + Cg backward, bf16
+    full = 2 * (T * d * 2)                   # X forward + G backward uncompressed
+    bytes_per_ms = link_mbps * 1e6 / 8 / 1e3
+    return {
+        "paper": "up to 99% compression (~100x, k = 40 at d = 4096) and up to 100x "
+                 "communication efficiency; 80 Mbps links matching 100 Gbps convergence "
+                 "(A10G / L4 GPUs, Sec. 1, Sec. 8.1)",
+        "wire_bytes_per_step": wire, "uncompressed_bytes_per_step": full,
+        "compression_ratio": full / wire, "compression_pct": 100.0 * (1 - wire / full),
+        "link_mbps": link_mbps,
+        "wire_ms_at_link": wire / bytes_per_ms, "uncompressed_ms_at_link": full / bytes_per_ms,
+        "codec_ms_per_step": codec_ms,
+        "note": "context, not the target: the codec's GPU time per step against the time its "
+                "output needs on the paper's slowest links"}
+
+
 # ---- our arm -------------------------------------------------------------------------
 
 def run_ours(args, world, rank, local, pg):
@@ -773,6 +795,7 @@ def run_ours(args, world, rank, local, pg):
             "next": nxt,
             "e2e": e2e_line,
             "graph": graph_line,
+            "paper_context": paper_context(T, d, k, ms),
             "gpu_launches": launches,
             "unique_ids": u,
             "wall_s_timed_region": wall,

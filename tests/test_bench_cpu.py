@@ -48,3 +48,11 @@ def test_algorithmic_bytes_of_the_large_stream():
     assert ab["sn_compress_fwd"] == ab["sn_decompress_fwd"] == 1371930624
     assert ab["sn_compress_bwd"] == ab["sn_decompress_bwd"] == 1087176704
     assert ab["sn_project_weight"] == 268435456
+
+
+def test_paper_context_of_the_large_stream():
+    ctx = _bench().paper_context(T=65536, d=8192, k=82, codec_ms=1.0)
+    assert ctx["wire_bytes_per_step"] == 2 * 65536 * 82 * 2
+    assert abs(ctx["compression_ratio"] - 8192 / 82) < 1e-9
+    assert abs(ctx["compression_pct"] - 100 * (1 - 82 / 8192)) < 1e-9
+    assert abs(ctx["wire_ms_at_link"] - 2 * 65536 * 82 * 2 / 1e4) < 1e-6      # 80 Mbps = 1e4 B/ms
