@@ -194,51 +194,94 @@ def max_over_ranks(pg, value, device=None):
 
 # ---- CPU oracle baseline ---------------------------------------------------------
 
+def _oracle_inputs(seed):
+    sys.path.insert(0, ROOT)
+    import oracle as O
+    from paper_2506_01260_gb300 import workloads as W
+    wl = W.WORKLOADS[WORKLOAD]
+    rng = np.random.default_rng(seed)
+    U = W.orthonormal_basis(wl.d, wl.k, rng).astype(np.float32)
+    return O.default(), W, rng, U, wl
+
+
+def _oracle_boundary(orc, W, rng, U, S, d):
+    """S tokens through the four boundary calls of the oracle; seconds."""
+    tok = W.to_bf16(0.02 * rng.standard_normal((S, d)))
+    pe = W.to_bf16(0.02 * rng.standard_normal((S, d)))
+    ids = np.arange(S, dtype=np.int32)
+    pos = np.arange(S, dtype=np.int32)
+    X = W.to_bf16(0.1 * rng.standard_normal((S, d)))
+    G = W.to_bf16(rng.standard_normal((S, d)))
+    t0 = time.perf_counter()
+    C, _, _ = orc.compress_fwd(X, ids, tok, U, S, pos_emb=pe, pos=pos)
+    orc.decompress_fwd(C, ids, tok, U, S, pos_emb=pe, pos=pos)
+    Cg, _, _ = orc.compress_bwd(G, U)
+    orc.decompress_bwd(Cg, U)
+    return time.perf_counter() - t0
+
+
+def _oracle_project(orc, W, rng, U, c, d):
+    """c columns of a [d, c] weight through the oracle's projection; seconds."""
+    Wc = W.to_bf16(0.02 * rng.standard_normal((d, c)))
+    t0 = time.perf_counter()
+    orc.project_weight(Wc, U)
+    return time.perf_counter() - t0
+
+
+def _oracle_worker(job):
+    """One process of the all-cores baseline: ("boundary", S) or ("project", c)."""
+    kind, size, seed = job
+    orc, W, rng, U, wl = _oracle_inputs(seed)
+    if size == 0:
+        return 0.0
+    if kind == "boundary":
+        return _oracle_boundary(orc, W, rng, U, size, wl.d)
+    return _oracle_project(orc, W, rng, U, size, wl.d)
+
+
 def cpu_oracle_step_time(target_s, seed=7):
     """Time the fp64 oracle on a bounded sample of the large-stream step and
     scale it to a full step: S tokens through the four boundary calls, plus c
     columns of W_o through the projection.  Returns (seconds per full step,
-    description of the sample)."""
-    import oracle as O
-    from paper_2506_01260_gb300 import workloads as W
-
-    wl = W.WORKLOADS[WORKLOAD]
-    orc = O.default()
-    rng = np.random.default_rng(seed)
-    d, k, n = wl.d, wl.k, wl.seq_len
-    U = W.orthonormal_basis(d, k, rng).astype(np.float32)
-
-    def boundary(S):
-        tok = W.to_bf16(0.02 * rng.standard_normal((S, d)))
-        pe = W.to_bf16(0.02 * rng.standard_normal((S, d)))
-        ids = np.arange(S, dtype=np.int32)
-        pos = np.arange(S, dtype=np.int32)
-        X = W.to_bf16(0.1 * rng.standard_normal((S, d)))
-        G = W.to_bf16(rng.standard_normal((S, d)))
-        t0 = time.perf_counter()
-        C, _, _ = orc.compress_fwd(X, ids, tok, U, S, pos_emb=pe, pos=pos)
-        orc.decompress_fwd(C, ids, tok, U, S, pos_emb=pe, pos=pos)
-        Cg, _, _ = orc.compress_bwd(G, U)
-        orc.decompress_bwd(Cg, U)
-        return time.perf_counter() - t0
-
-    def project(c):
-        Wc = W.to_bf16(0.02 * rng.standard_normal((d, c)))
-        t0 = time.perf_counter()
-        orc.project_weight(Wc, U)
-        return time.perf_counter() - t0
-
-    t_probe = boundary(8) / 8
+    description of the sample, seconds spent, (S, c))."""
+    orc, W, rng, U, wl = _oracle_inputs(seed)
+    d = wl.d
+    t_probe = _oracle_boundary(orc, W, rng, U, 8, d) / 8
     S = int(max(8, min(wl.T, 0.85 * target_s / max(t_probe, 1e-9))))
-    tb = boundary(S)
-    p_probe = project(4) / 4
+    tb = _oracle_boundary(orc, W, rng, U, S, d)
+    p_probe = _oracle_project(orc, W, rng, U, 4, d) / 4
     c = int(max(4, min(W_O_SHAPE[1], 0.15 * target_s / max(p_probe, 1e-9))))
-    tp = project(c)
+    tp = _oracle_project(orc, W, rng, U, c, d)
     step = tb * wl.T / S + tp * W_O_SHAPE[1] / c
     desc = ("fp64 oracle, 1 thread: %d of %d tokens through compress_fwd+decompress_fwd+"
             "compress_bwd+decompress_bwd (%.1f s) and %d of %d W_o columns through "
             "project_weight (%.1f s), scaled to one full step" % (S, wl.T, tb, c, W_O_SHAPE[1], tp))
-    return step, desc, tb + tp
+    return step, desc, tb + tp, (S, c)
+
+
+def cpu_oracle_step_time_all_cores(S, c, seed=11):
+    """The same sample as cpu_oracle_step_time split over every host core: one
+    spawned process per core takes an equal share of the S tokens, then of the
+    c columns (the oracle itself is single-threaded; the shards are independent
+    rows and columns).  A phase takes as long as its slowest process's oracle
+    calls (each process builds its inputs first, untimed, like the one-thread
+    sample); scaled to one full step."""
+    import multiprocessing as mp
+    from paper_2506_01260_gb300 import workloads as W
+    wl = W.WORKLOADS[WORKLOAD]
+    n = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    n = max(1, int(n))
+    ctx = mp.get_context("spawn")
+    with ctx.Pool(n) as pool:
+        tb = max(pool.map(_oracle_worker,
+                          [("boundary", S // n + (i < S % n), seed + i) for i in range(n)]))
+        tp = max(pool.map(_oracle_worker,
+                          [("project", c // n + (i < c % n), seed + i) for i in range(n)]))
+    step = tb * wl.T / S + tp * W_O_SHAPE[1] / c
+    desc = ("fp64 oracle in %d processes (one per host core): the same %d tokens (slowest "
+            "process %.2f s) and %d W_o columns (slowest %.2f s), scaled to one full step"
+            % (n, S, tb, c, tp))
+    return step, desc, n
 
 
 def run_reference(args, world, rank):
@@ -248,7 +291,7 @@ def run_reference(args, world, rank):
     steps = []
     desc = None
     for i in range(args.warmup + args.steps):
-        st, desc, _ = cpu_oracle_step_time(max(1.0, args.cpu_seconds / 4), seed=100 + i)
+        st, desc, _, _ = cpu_oracle_step_time(max(1.0, args.cpu_seconds / 4), seed=100 + i)
         if i >= args.warmup:
             steps.append(st)
     from paper_2506_01260_gb300 import workloads as W
@@ -772,9 +815,15 @@ def run_ours(args, world, rank, local, pg):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline and args.workload == WORKLOAD:
-        st, desc, _ = cpu_oracle_step_time(args.cpu_seconds)
+        st, desc, _, (S, c) = cpu_oracle_step_time(args.cpu_seconds)
         cpu = {"value": T / st, "unit": "tokens/s", "cores": 1, "kind": "oracle",
                "sample": desc}
+        try:
+            st_all, desc_all, n_all = cpu_oracle_step_time_all_cores(S, c)
+            cpu["all_cores"] = {"value": T / st_all, "unit": "tokens/s", "cores": n_all,
+                                "sample": desc_all}
+        except Exception as exc:          # a host without spawnable workers
+            cpu["all_cores"] = {"unavailable": repr(exc)[:200]}
 
     if rank == 0:
         line = {
