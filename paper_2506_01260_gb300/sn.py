@@ -112,6 +112,22 @@ def _ptr(t):
     return None if t is None else ctypes.c_void_p(t.data_ptr())
 
 
+def _check_rows(T, seq_len, d, pos_emb, pos, width=None):
+    """pos has T entries and the positional table seq_len rows of `width`
+    (d, or k for a projected table): the kernels index them without bounds
+    information, so a short table is refused here."""
+    if pos is not None and pos.shape != (T,):
+        raise ValueError("pos must have shape [T]")
+    if pos_emb is not None and (pos_emb.dim() != 2 or pos_emb.shape[0] < seq_len or
+                                pos_emb.shape[1] != (d if width is None else width)):
+        raise ValueError("the positional table must have seq_len rows of the right width")
+
+
+def _check_out(out, shape):
+    if tuple(out.shape) != tuple(shape):
+        raise ValueError("out must have shape %s" % (tuple(shape),))
+
+
 def _need(t, name, dtype=None, contiguous=True):
     if not isinstance(t, torch.Tensor):
         raise TypeError("%s must be a torch.Tensor" % name)
@@ -182,9 +198,11 @@ def sn_compress_fwd(basis, X, ids, tok_emb, seq_len, pos_emb=None, pos=None, out
     T = X.shape[0]
     if X.shape != (T, basis.d) or ids.shape != (T,) or tok_emb.shape[1] != basis.d:
         raise ValueError("shape mismatch")
+    _check_rows(T, seq_len, basis.d, pos_emb, pos)
     if out is None:
         out = torch.empty(T, basis.k, dtype=X.dtype, device=X.device)
     _need(out, "out", X.dtype)
+    _check_out(out, (T, basis.k))
     _check(_lib.sn_compress_fwd(basis.handle, _dtype(X), _ptr(X), _ptr(ids), _ptr(pos), T,
                                 seq_len, _ptr(tok_emb), tok_emb.shape[0], _ptr(pos_emb),
                                 _ptr(out), _stream(stream)), "sn_compress_fwd")
@@ -227,11 +245,13 @@ def sn_compress_fwd_projected(basis, X, ids, TU, seq_len, PU=None, pos=None, out
     if pos is not None:
         _need(pos, "pos", torch.int32)
     T = X.shape[0]
-    if X.shape != (T, basis.d) or ids.shape != (T,) or TU.shape[1] != basis.k:
+    if X.shape != (T, basis.d) or ids.shape != (T,) or TU.dim() != 2 or TU.shape[1] != basis.k:
         raise ValueError("shape mismatch")
+    _check_rows(T, seq_len, basis.d, PU, pos, width=basis.k)
     if out is None:
         out = torch.empty(T, basis.k, dtype=X.dtype, device=X.device)
     _need(out, "out", X.dtype)
+    _check_out(out, (T, basis.k))
     _check(_lib.sn_compress_fwd_projected(basis.handle, _dtype(X), _ptr(X), _ptr(ids), _ptr(pos),
                                           T, seq_len, _ptr(TU), TU.shape[0], _ptr(PU), _ptr(out),
                                           _stream(stream)), "sn_compress_fwd_projected")
@@ -433,9 +453,11 @@ def sn_decompress_fwd(basis, C, ids, tok_emb, seq_len, pos_emb=None, pos=None, o
     T = C.shape[0]
     if C.shape != (T, basis.k) or ids.shape != (T,) or tok_emb.shape[1] != basis.d:
         raise ValueError("shape mismatch")
+    _check_rows(T, seq_len, basis.d, pos_emb, pos)
     if out is None:
         out = torch.empty(T, basis.d, dtype=C.dtype, device=C.device)
     _need(out, "out", C.dtype)
+    _check_out(out, (T, basis.d))
     _check(_lib.sn_decompress_fwd(basis.handle, _dtype(C), _ptr(C), _ptr(ids), _ptr(pos), T,
                                   seq_len, _ptr(tok_emb), tok_emb.shape[0], _ptr(pos_emb),
                                   _ptr(out), _stream(stream)), "sn_decompress_fwd")
@@ -451,6 +473,7 @@ def sn_compress_bwd(basis, G, out=None, stream=None):
     if out is None:
         out = torch.empty(T, basis.k, dtype=G.dtype, device=G.device)
     _need(out, "out", G.dtype)
+    _check_out(out, (T, basis.k))
     _check(_lib.sn_compress_bwd(basis.handle, _dtype(G), _ptr(G), T, _ptr(out), _stream(stream)),
            "sn_compress_bwd")
     return out
@@ -465,6 +488,7 @@ def sn_decompress_bwd(basis, C, out=None, stream=None):
     if out is None:
         out = torch.empty(T, basis.d, dtype=C.dtype, device=C.device)
     _need(out, "out", C.dtype)
+    _check_out(out, (T, basis.d))
     _check(_lib.sn_decompress_bwd(basis.handle, _dtype(C), _ptr(C), T, _ptr(out),
                                   _stream(stream)), "sn_decompress_bwd")
     return out

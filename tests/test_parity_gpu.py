@@ -469,3 +469,37 @@ def test_host_pointers_are_refused(sn):
     sn.sn_compress_fwd(basis, X, ids, tok, n, out=C)  # device memory still works
     sn.sn_check_errors(basis)
     basis.destroy()
+
+
+def test_binding_refuses_short_tables_and_wrong_outputs(sn):
+    """The kernels index the positional table by position and write T rows of
+    the output without bounds information, so the binding refuses a positional
+    table with fewer than seq_len rows, a pos array of the wrong length and an
+    output of the wrong shape before anything is launched."""
+    T, n, d, k, vocab = 256, 128, 256, 8, 1024
+    U = torch.linalg.qr(torch.randn(d, k, dtype=torch.float64))[0].float().contiguous().cuda()
+    basis = sn.Basis(U)
+    X = torch.zeros(T, d, dtype=torch.bfloat16, device="cuda")
+    ids = torch.zeros(T, dtype=torch.int32, device="cuda")
+    tok = torch.zeros(vocab, d, dtype=torch.bfloat16, device="cuda")
+    pe = torch.zeros(n, d, dtype=torch.bfloat16, device="cuda")
+    C = torch.zeros(T, k, dtype=torch.bfloat16, device="cuda")
+    launches = sn.sn_launch_count()
+    bad_calls = [
+        lambda: sn.sn_compress_fwd(basis, X, ids, tok, n + 1, pos_emb=pe),           # short table
+        lambda: sn.sn_decompress_fwd(basis, C, ids, tok, n + 1, pos_emb=pe),
+        lambda: sn.sn_compress_fwd(basis, X, ids, tok, n, pos_emb=pe[:, :128]),      # narrow table
+        lambda: sn.sn_compress_fwd(basis, X, ids, tok, n, pos_emb=pe,
+                                   pos=ids[:100]),                                    # short pos
+        lambda: sn.sn_compress_fwd(basis, X, ids, tok, n, out=C[:100]),               # short out
+        lambda: sn.sn_decompress_fwd(basis, C, ids, tok, n, out=X[:, :128]),
+        lambda: sn.sn_compress_bwd(basis, X, out=C[:, :4]),
+        lambda: sn.sn_decompress_bwd(basis, C, out=X[:10]),
+    ]
+    for call in bad_calls:
+        with pytest.raises(ValueError):
+            call()
+    assert sn.sn_launch_count() == launches
+    sn.sn_compress_fwd(basis, X, ids, tok, n, pos_emb=pe, out=C)     # the valid call runs
+    sn.sn_check_errors(basis)
+    basis.destroy()
