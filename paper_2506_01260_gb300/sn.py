@@ -218,6 +218,7 @@ def sn_project_tables(basis, tok_emb, pos_emb=None, TU=None, PU=None, stream=Non
     if TU is None:
         TU = torch.empty(V, basis.k, dtype=torch.float32, device=tok_emb.device)
     _need(TU, "TU", torch.float32)
+    _check_out(TU, (V, basis.k))
     n = 0
     if pos_emb is not None:
         _need(pos_emb, "pos_emb", tok_emb.dtype)
@@ -227,6 +228,7 @@ def sn_project_tables(basis, tok_emb, pos_emb=None, TU=None, PU=None, stream=Non
         if PU is None:
             PU = torch.empty(n, basis.k, dtype=torch.float32, device=tok_emb.device)
         _need(PU, "PU", torch.float32)
+        _check_out(PU, (n, basis.k))
     else:
         PU = None
     _check(_lib.sn_project_tables(basis.handle, _dtype(tok_emb), _ptr(tok_emb), V, _ptr(pos_emb),
@@ -267,9 +269,11 @@ def sn_build_ts(basis, tok_emb, out=None, workspace=None, stream=None):
     if out is None:
         out = torch.empty_like(tok_emb)
     _need(out, "out", tok_emb.dtype)
+    _check_out(out, (V, basis.d))
     nbytes = sn_wire_bytes(basis, tok_emb.dtype, V)
     if workspace is None:
         workspace = torch.empty(max(16, nbytes), dtype=torch.uint8, device=tok_emb.device)
+    _need(workspace, "workspace")
     _check(_lib.sn_build_ts(basis.handle, _dtype(tok_emb), _ptr(tok_emb), V, _ptr(out),
                             _ptr(workspace), workspace.numel() * workspace.element_size(),
                             _stream(stream)), "sn_build_ts")
@@ -295,8 +299,11 @@ def sn_grassmann_accumulate(basis, G, Cg, M, workspace=None, stream=None):
     if workspace is None:
         workspace = torch.empty(max(256, sn_grassmann_workspace(basis, T)[0]), dtype=torch.uint8,
                                 device=G.device)
+    _need(workspace, "workspace")
     _check(_lib.sn_grassmann_accumulate(basis.handle, SN_BF16, _ptr(G), _ptr(Cg), T, _ptr(M),
-                                        _ptr(workspace), workspace.numel(), _stream(stream)),
+                                        _ptr(workspace),
+                                        workspace.numel() * workspace.element_size(),
+                                        _stream(stream)),
            "sn_grassmann_accumulate")
     return M
 
@@ -322,11 +329,14 @@ def sn_grassmann_step(basis, M, K, eta, out=None, workspace=None, stream=None):
     if out is None:
         out = torch.empty_like(M)
     _need(out, "out", torch.float32)
+    _check_out(out, (basis.d, basis.k))
     if workspace is None:
         workspace = torch.empty(max(256, sn_grassmann_workspace(basis, 1)[1]), dtype=torch.uint8,
                                 device=M.device)
+    _need(workspace, "workspace")
     _check(_lib.sn_grassmann_step(basis.handle, _ptr(M), int(K), float(eta), _ptr(out),
-                                  _ptr(workspace), workspace.numel(), _stream(stream)),
+                                  _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                  _stream(stream)),
            "sn_grassmann_step")
     return out
 
@@ -343,6 +353,7 @@ def sn_adamw_rowconst(W, grad, M, V, step, lr, beta1=0.9, beta2=0.999, eps=1e-8,
     rows, cols = W.shape
     if workspace is None:
         workspace = torch.empty(cols, dtype=torch.float32, device=W.device)
+    _need(workspace, "workspace")
     _check(_lib.sn_adamw_rowconst(_dtype(grad), _ptr(W), _ptr(grad), _ptr(M), _ptr(V), rows, cols,
                                   int(step), float(lr), float(beta1), float(beta2), float(eps),
                                   float(lam), _ptr(workspace),
@@ -372,8 +383,12 @@ def sn_topk_restore(vals, cols, d, out=None, stream=None):
     _need(vals, "values", torch.bfloat16)
     _need(cols, "cols", torch.int16)
     T, kk = vals.shape
+    if cols.shape != vals.shape:
+        raise ValueError("values and cols must have the same shape [T, kk]")
     if out is None:
         out = torch.empty(T, d, dtype=torch.bfloat16, device=vals.device)
+    _need(out, "out", torch.bfloat16)
+    _check_out(out, (T, d))
     _check(_lib.sn_topk_restore(_ptr(vals), _ptr(cols), T, d, kk, _ptr(out), _stream(stream)),
            "sn_topk_restore")
     return out
@@ -400,8 +415,12 @@ def sn_sign_restore(bits, scale, d, out=None, stream=None):
     _need(bits, "bits", torch.int32)
     _need(scale, "scale", torch.float32)
     T = scale.shape[0]
+    if scale.dim() != 1 or bits.shape != (T, (d + 31) // 32):
+        raise ValueError("bits must be [T, ceil(d/32)] and scale [T]")
     if out is None:
         out = torch.empty(T, d, dtype=torch.bfloat16, device=scale.device)
+    _need(out, "out", torch.bfloat16)
+    _check_out(out, (T, d))
     _check(_lib.sn_sign_restore(_ptr(bits), _ptr(scale), T, d, _ptr(out), _stream(stream)),
            "sn_sign_restore")
     return out
@@ -433,8 +452,12 @@ def sn_quant_restore(codes, scale, fmt, out=None, stream=None):
     _need(codes, "codes", torch.uint8)
     _need(scale, "scale", torch.float32)
     T, d = codes.shape
+    if scale.shape != (T,):
+        raise ValueError("scale must be [T]")
     if out is None:
         out = torch.empty(T, d, dtype=torch.bfloat16, device=codes.device)
+    _need(out, "out", torch.bfloat16)
+    _check_out(out, (T, d))
     _check(_lib.sn_quant_restore(_ptr(codes), _ptr(scale), T, d, QUANT_FORMATS[fmt], _ptr(out),
                                  _stream(stream)), "sn_quant_restore")
     return out
@@ -512,11 +535,13 @@ def sn_project_weight(basis, W, out=None, workspace=None, stream=None):
     ld = W.stride(0)
     if out is None:
         out = torch.empty_like(W)
+    _need(out, "out", W.dtype, contiguous=False)
     if out.stride() != W.stride() or out.shape != W.shape:
         raise ValueError("out must have W's shape and strides")
     need = sn_project_weight_workspace(basis, W.dtype, cols)
     if workspace is None:
         workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=W.device)
+    _need(workspace, "workspace")
     _check(_lib.sn_project_weight(basis.handle, _dtype(W), _ptr(W), rows, cols, ld, _ptr(out),
                                   _ptr(workspace), workspace.numel() * workspace.element_size(),
                                   _stream(stream)), "sn_project_weight")
@@ -529,6 +554,7 @@ def sn_project_weight_noalloc(basis, W, out, stream=None):
     instead of a workspace, and the caller provides `out` (may be W).  bf16
     only.  Calls that overlap on the GPU share the scratch and race."""
     _need(W, "W", torch.bfloat16, contiguous=False)
+    _need(out, "out", torch.bfloat16, contiguous=False)
     if W.dim() != 2 or W.shape[0] != basis.d or W.stride(1) != 1:
         raise ValueError("W must be [d, cols] with unit column stride")
     if out.stride() != W.stride() or out.shape != W.shape or out.dtype != W.dtype:
