@@ -33,12 +33,12 @@
  *   - Only sn_basis_create allocates (and sn_basis_destroy frees); no other
  *     call allocates memory or falls back to the CPU.  A basis holds two
  *     scratch areas of (SM count) x 128 x (k rounded up to 16) floats that the
- *     bf16 compress calls use for the partial sums of their last-round row
- *     tiles: one for the forward compress calls (sn_compress_fwd,
- *     sn_compress_fwd_projected), one for sn_compress_bwd.  Forward calls on
- *     one basis must therefore not overlap each other in time (other streams,
- *     other host threads), nor backward calls each other; a forward and a
- *     backward call may.
+ *     bf16 contractions use for the partial sums of their last-round row
+ *     tiles: one for the forward calls (sn_compress_fwd,
+ *     sn_compress_fwd_projected, sn_project_tables), one for sn_compress_bwd.
+ *     Forward calls on one basis must therefore not overlap each other in time
+ *     (other streams, other host threads), nor backward calls each other; a
+ *     forward and a backward call may.
  *   - Every wait inside a kernel is bounded; a wait that expires records
  *     SN_ERR_TIMEOUT in the error word and the kernel returns.
  */

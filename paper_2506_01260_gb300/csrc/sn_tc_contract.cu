@@ -226,7 +226,7 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
             }
             tc_fence_after();
             const uint32_t taddr = tmem + b * p.acc_stride + ((uint32_t)(32 * q) << 16);
-            if (MODE != CMODE_W && MODE != CMODE_GF && sp.tail) {
+            if (MODE != CMODE_W && sp.tail) {
                 // a d-range of a tail tile: fp32 partial row, summed by k_sum_tail
                 float *dst = p.Ptail +
                              (((int64_t)(tile - (p.ntiles - p.tail_tiles)) * p.tail_splits + split) *

@@ -227,7 +227,8 @@ int current_device()
 }  // namespace
 }  // namespace tc
 
-// Last-round split of the compress contractions.  With one CTA per SM a grid
+// Last-round split of the compress contractions and of the fp32 table
+// projection.  With one CTA per SM a grid
 // whose last round holds rem < sms / 2 row tiles leaves most SMs idle for a
 // whole tile; those tiles instead run as s = min(4, sms / rem) items over
 // d-ranges of at least 8 chunks, writing fp32 partials to the basis' scratch,
@@ -255,6 +256,7 @@ void plan_tail(tc::ContractParams &p, int sms, float *scratch, int cap)
 // C rows of the split tiles: the sum of their d-range partials (minus the
 // projected embedding rows in XP mode), rounded once to bf16; a row with an
 // invalid id or position is written as zeros and flagged (X and XP modes).
+// The fp32 table projection (GF mode) keeps the sum in fp32.
 // Grid (tail tiles, 128 / 8): one warp per row, the lanes across its k columns.
 __global__ void __launch_bounds__(256) k_sum_tail(const __grid_constant__ tc::ContractParams p,
                                                   int mode)
@@ -268,7 +270,7 @@ __global__ void __launch_bounds__(256) k_sum_tail(const __grid_constant__ tc::Co
         return;
     bool bad = false;
     int id = 0, ps = 0;
-    if (mode != CMODE_G) {
+    if (mode != CMODE_G && mode != CMODE_GF) {
         id = p.ids[row];
         bad = id < 0 || id >= p.vocab;
         if (p.has_pe) {
@@ -289,7 +291,10 @@ __global__ void __launch_bounds__(256) k_sum_tail(const __grid_constant__ tc::Co
             if (p.has_pe)
                 v -= p.PU[(int64_t)ps * p.k + j];
         }
-        p.C[row * p.k + j] = __float2bfloat16_rn(bad ? 0.f : v);
+        if (mode == CMODE_GF)
+            p.Cf[row * p.k + j] = v;            // projected table rows stay fp32
+        else
+            p.C[row * p.k + j] = __float2bfloat16_rn(bad ? 0.f : v);
     }
 }
 
@@ -385,7 +390,11 @@ cudaError_t tc_contract_f32(const sn_basis &b, const __nv_bfloat16 *A, int64_t r
         return cudaErrorInvalidValue;
     p.Cf = out;
     p.stages = contract_stages(CMODE_GF, b.n_pad, b.k, 0);
-    return launch_contract(CMODE_GF, p, std::min(p.ntiles, sm_count(current_device())), s);
+    // short tables (a positional table of a few thousand rows) split their
+    // last round over d like the compress calls, on the forward scratch
+    const int sms = sm_count(current_device());
+    plan_tail(p, sms, b.tail[0], b.tail_cap);
+    return launch_compress(CMODE_GF, p, sms, s);
 }
 
 cudaError_t tc_compress_projected(const sn_basis &b, const __nv_bfloat16 *X, const int32_t *ids,
