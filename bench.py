@@ -852,6 +852,11 @@ def run_ours(args, world, rank, local, pg):
                         "compute_stream_wait": seg["wire_wait"]},
             "boundary_hbm_gbs": sum(ab[nm] for nm in names) / (
                 sum(seg[nm] for nm in names) / 1e3) / 1e9,
+            # tokens/s of each round trip alone (compress + decompress), beside the
+            # whole step's `value`
+            "round_trip_tokens_per_s": {
+                "fwd": world * T / ((seg["sn_compress_fwd"] + seg["sn_decompress_fwd"]) / 1e3),
+                "bwd": world * T / ((seg["sn_compress_bwd"] + seg["sn_decompress_bwd"]) / 1e3)},
             "next": nxt,
             "e2e": e2e_line,
             "graph": graph_line,
