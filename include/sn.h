@@ -138,8 +138,10 @@ sn_status sn_project_weight(sn_basis_t basis, sn_dtype dtype, const void *W, int
  * Arguments, layout and results are those of sn_project_weight; bf16 only.
  * Returns SN_ERR_UNSUPPORTED for SN_F32 and when sn_project_weight_workspace
  * for `cols` exceeds 32 MiB.  The first call on a device (with that device
- * current) looks up the array's device address; make that first call before
- * any stream capture.  All calls share the one array: calls whose executions
+ * current) looks up the array's device address in the current CUDA context;
+ * a call made under another context of the device (after cudaDeviceReset, or
+ * under a caller's own context) looks it up again.  Make the first call in
+ * each context before any stream capture.  All calls share the one array: calls whose executions
  * overlap on the GPU (other streams, other host threads) race and corrupt each
  * other's results, so order them on one stream.  Each call writes every
  * scratch element it reads before reading it; nothing is kept between calls. */

@@ -49,6 +49,14 @@ def accumulate(M, G, U):
     return np.asarray(M, np.float64) + G.T @ (G @ np.asarray(U, np.float64))
 
 
+def accumulate_rows(M_rows, G, U, rows):
+    """Rows `rows` of M + G^T (G U) alone: M_rows + G[:, rows]^T (G U).  The
+    same sum as `accumulate`, for checking a large accumulation on sampled
+    rows (G U still needs every column of G)."""
+    G = np.asarray(G, np.float64)
+    return np.asarray(M_rows, np.float64) + G[:, rows].T @ (G @ np.asarray(U, np.float64))
+
+
 def euclidean_grad(M, K):
     """-2 S U with S U = M / K."""
     return -2.0 * np.asarray(M, np.float64) / K

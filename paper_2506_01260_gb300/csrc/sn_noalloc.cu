@@ -9,7 +9,11 @@
 // kNoallocScratchBytes of it until the process exits.  Host code cannot use
 // the array's name as a device address, so the first call on each device
 // (with that device current) looks the address up with cudaGetSymbolAddress;
-// later calls reuse it.
+// later calls in the same CUDA context reuse it.  The address belongs to the
+// context it was looked up in, so it is cached together with that context and
+// looked up again when the device's current context is a different one (after
+// cudaDeviceReset, or under a caller's own non-primary context).
+#include <cuda.h>
 #include <mutex>
 
 #include "sn_internal.cuh"
@@ -23,9 +27,29 @@ static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocScratch
 
 std::mutex g_noalloc_mu;
 void *g_noalloc_ptr[kMaxDevices];
+CUcontext g_noalloc_ctx[kMaxDevices];
 
-// Device address of the scratch array on the current device (set-up on the
-// first call per device).
+typedef CUresult (*CtxGetCurrentFn)(CUcontext *);
+
+// The driver's cuCtxGetCurrent, reached through the runtime (the library does
+// not link the driver library itself).
+CtxGetCurrentFn ctx_get_current()
+{
+    static CtxGetCurrentFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = (CtxGetCurrentFn)f;
+    });
+    return fn;
+}
+
+// Device address of the scratch array on the current device, in the current
+// context (set-up on the first call per device and context).
 sn_status noalloc_scratch(void **out)
 {
     int dev = -1;
@@ -33,12 +57,20 @@ sn_status noalloc_scratch(void **out)
         return SN_ERR_CUDA;
     if (dev < 0 || dev >= kMaxDevices)
         return SN_ERR_UNSUPPORTED;
+    CtxGetCurrentFn get = ctx_get_current();
+    CUcontext ctx = nullptr;
+    if (!get || get(&ctx) != CUDA_SUCCESS)
+        return SN_ERR_CUDA;
     std::lock_guard<std::mutex> lock(g_noalloc_mu);
-    if (!g_noalloc_ptr[dev]) {
+    if (!ctx || !g_noalloc_ptr[dev] || g_noalloc_ctx[dev] != ctx) {
         void *p = nullptr;
         if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p)
             return SN_ERR_CUDA;
+        // the lookup makes the device's primary context current if none was
+        if (!ctx && (get(&ctx) != CUDA_SUCCESS || !ctx))
+            return SN_ERR_CUDA;
         g_noalloc_ptr[dev] = p;
+        g_noalloc_ctx[dev] = ctx;
     }
     *out = g_noalloc_ptr[dev];
     return SN_OK;

@@ -339,9 +339,10 @@ __device__ __forceinline__ void prefetch_l2_range(const void *p, int bytes)
 
 // ---- cp.async: 16-byte global -> shared copies issued per thread -------------
 // Used for row gathers: each thread places its chunks directly at their
-// swizzled positions.  Completion is observed with wait_group by the issuing
-// thread, which then fences toward the async proxy before arriving on the
-// stage's mbarrier.
+// swizzled positions and hands their completion to the stage's mbarrier with
+// cp_async_arrive (cp.async.mbarrier.arrive.noinc); the consumer that waits on
+// that barrier fences toward the async proxy before the tensor cores or a TMA
+// store read the rows.
 // Copies `src_bytes` (0 or 16) bytes and zero-fills the rest of the 16.
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, uint32_t src_bytes)
 {

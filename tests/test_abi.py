@@ -49,9 +49,9 @@ def test_status_strings(lib):
     f = lib.sn_status_string
     f.restype = ctypes.c_char_p
     f.argtypes = [ctypes.c_int]
-    names = [f(i).decode() for i in range(7)]
+    names = [f(i).decode() for i in range(8)]
     assert names == ["SN_OK", "SN_ERR_INVALID_ARG", "SN_ERR_ALIGNMENT", "SN_ERR_UNSUPPORTED",
-                     "SN_ERR_BAD_ID", "SN_ERR_TIMEOUT", "SN_ERR_CUDA"]
+                     "SN_ERR_BAD_ID", "SN_ERR_TIMEOUT", "SN_ERR_CUDA", "SN_ERR_NUMERIC"]
     assert f(99).decode() == "SN_ERR_UNKNOWN"
 
 

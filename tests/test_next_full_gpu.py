@@ -3,13 +3,15 @@ calls the benchmark times, on samples the fp64 oracles compute one by one:
 - the projected-table compress (Eq. subtract with T_fixed U, P U): sampled
   tokens against the plain compress of the oracle;
 - the Grassmann accumulation M = G^T (G U) over all 65536 tokens (Sec. 6):
-  sampled rows of M, the oracle's G U formed in fp64 a chunk of tokens at a
-  time;
+  sampled rows of M against the Grassmann oracle's sum, fed a chunk of tokens
+  at a time;
 - the row-constant AdamW step on W_o [8192, 8192] (Sec. 5): sampled columns
   (each column's rate depends only on that column);
 - the top-k, sign and 8-bit comparators on X (Sec. 8): sampled rows.
-Bars as everywhere: 1e-2 relative Frobenius error for bf16 results, 1e-5 for
-fp32 ones, exact for selected columns, sign bits and 8-bit codes."""
+Bars as everywhere: 1e-2 relative Frobenius error and 3e-2 on the worst row for
+bf16 results (the Grassmann accumulation takes the bf16 bar: it reads the bf16
+G and the tensor cores' bf16 products), 1e-5 for fp32 ones, exact for selected
+columns, sign bits and 8-bit codes."""
 import importlib.util
 import os
 
@@ -17,7 +19,7 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_util import TOL, host, rel_fro, widen
+from gpu_util import assert_parity, host, widen
 from paper_2506_01260_gb300 import workloads as W
 
 pytestmark = pytest.mark.gpu
@@ -64,11 +66,12 @@ def test_projected_compress_full_size(sn, oracle, large):
                                      inp["U"].cpu().numpy(), len(rows), pos_emb=pe,
                                      pos=np.arange(len(rows), dtype=np.int32))
     assert st == 0
-    assert rel_fro(host(C[rt]), C64) <= TOL["bf16"]
+    assert_parity(host(C[rt]), C64, "bf16")
     basis.destroy()
 
 
 def test_grassmann_accumulate_full_size(sn, large):
+    g = _load("grassmann")
     wl, inp = large
     basis = sn.Basis(inp["U"])
     G = inp["G"]
@@ -76,14 +79,13 @@ def test_grassmann_accumulate_full_size(sn, large):
     M = torch.zeros(wl.d, wl.k, dtype=torch.float32, device="cuda")
     sn.sn_grassmann_accumulate(basis, G, Cg, M)
     sn.sn_check_errors(basis)
-    U64 = inp["U"].double()
-    cols = torch.from_numpy(_rows(wl.d, 22, n=24)).cuda()
-    ref = torch.zeros(len(cols), wl.k, dtype=torch.float64, device="cuda")
-    for t0 in range(0, wl.T, 4096):                   # G U in fp64, a chunk of tokens at a time
-        Gc = G[t0:t0 + 4096].double()
-        ref += Gc[:, cols].t() @ (Gc @ U64)
-    got = M[cols].double()
-    assert float((got - ref).norm() / ref.norm()) <= 1e-2
+    U64 = inp["U"].double().cpu().numpy()
+    rows = _rows(wl.d, 22, n=24)
+    ref = np.zeros((len(rows), wl.k))
+    for t0 in range(0, wl.T, 4096):       # the oracle's sum, a chunk of tokens at a time
+        ref = g.accumulate_rows(ref, widen(host(G[t0:t0 + 4096])), U64, rows)
+    got = M[torch.from_numpy(rows).cuda()].cpu().numpy()
+    assert_parity(got, ref, "bf16")
     basis.destroy()
 
 

@@ -61,6 +61,17 @@ def pin_accumulation(g):
             and np.allclose(g.accumulation_matrix(Gs), S, rtol=1e-12, atol=1e-12))
 
 
+def pin_accumulation_rows(g):
+    rng, Gs, U = problem(9)
+    rows = np.array([0, 5, 6, 23])
+    M0 = rng.standard_normal((len(rows), U.shape[1]))
+    Mr = M0.copy()
+    for G in Gs:
+        Mr = g.accumulate_rows(Mr, G, U, rows)
+    S = sum(G.T @ G for G in Gs)                     # brute force, written out here
+    return np.allclose(Mr, M0 + (S @ U)[rows], rtol=1e-12, atol=1e-12)
+
+
 def pin_loss_trace(g):
     _, Gs, U = problem(3)
     S = sum(G.T @ G for G in Gs) / len(Gs)
@@ -120,7 +131,7 @@ def pin_converges_to_top_eigenspace(g):
     return np.max(np.abs(U @ U.T - P_top)) <= 1e-6
 
 
-PINS = [pin_finite_difference, pin_accumulation, pin_loss_trace, pin_tangent, pin_retraction,
+PINS = [pin_finite_difference, pin_accumulation, pin_accumulation_rows, pin_loss_trace, pin_tangent, pin_retraction,
         pin_descent, pin_in_subspace_fixed_point, pin_converges_to_top_eigenspace]
 
 
@@ -138,6 +149,10 @@ MUTANTS = {
                                "return G.T @ (G @ np.asarray(U, np.float64))"),
     "accumulate_gram_of_rows": ("return np.asarray(M, np.float64) + G.T @ (G @ np.asarray(U, np.float64))",
                                 "return np.asarray(M, np.float64) + (G.T @ G).T @ np.asarray(U, np.float64) * (G.shape[0] / G.shape[1])"),
+    "rows_forget_sum": ("return np.asarray(M_rows, np.float64) + G[:, rows].T @ (G @ np.asarray(U, np.float64))",
+                        "return G[:, rows].T @ (G @ np.asarray(U, np.float64))"),
+    "rows_transposed": ("return np.asarray(M_rows, np.float64) + G[:, rows].T @ (G @ np.asarray(U, np.float64))",
+                        "return np.asarray(M_rows, np.float64) + (G.T @ (G @ np.asarray(U, np.float64)))[rows[::-1]]"),
     "tangent_missing": ("return g - U @ (U.T @ g)", "return g"),
     "tangent_sign": ("return g - U @ (U.T @ g)", "return g + U @ (U.T @ g)"),
     "retract_no_sign_fix": ("return Q * s", "return Q"),

@@ -13,7 +13,7 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_util import TOL, dev, dtname, guarded, guards_intact, host, rel_fro, widen
+from gpu_util import assert_parity, dev, dtname, guarded, guards_intact, host, widen
 from paper_2506_01260_gb300 import workloads as W
 
 pytestmark = pytest.mark.gpu
@@ -63,10 +63,10 @@ def test_forward_round_trip(sn, oracle, case, dtype):
     _, C64, st = oracle.compress_fwd(inp["X"], inp["ids"], inp["tok_emb"], inp["U"], n,
                                      pos_emb=inp["pos_emb"])
     assert st == 0
-    assert rel_fro(host(C), C64) <= TOL[dtype]
+    assert_parity(host(C), C64, dtype)
     _, X64, _ = oracle.decompress_fwd(host(C), inp["ids"], inp["tok_emb"], inp["U"], n,
                                       pos_emb=inp["pos_emb"])
-    assert rel_fro(host(Xr), X64) <= TOL[dtype]
+    assert_parity(host(Xr), X64, dtype)
     # wire layout: C is a contiguous [T, k] slab, T*k elements, nothing else
     assert sn.sn_wire_bytes(basis, tdt, T) == T * k * (2 if dtype == "bf16" else 4)
     basis.destroy()
@@ -86,9 +86,9 @@ def test_backward_round_trip(sn, oracle, case, dtype):
     sn.sn_check_errors(basis)
     assert guards_intact(fullC) and guards_intact(fullG)
     _, C64, _ = oracle.compress_bwd(inp["G"], inp["U"])
-    assert rel_fro(host(C), C64) <= TOL[dtype]
+    assert_parity(host(C), C64, dtype)
     _, G64, _ = oracle.decompress_bwd(host(C), inp["U"])
-    assert rel_fro(host(Gr), G64) <= TOL[dtype]
+    assert_parity(host(Gr), G64, dtype)
     basis.destroy()
 
 
@@ -107,14 +107,14 @@ def test_explicit_positions_and_no_positional_table(sn, oracle, dtype):
     sn.sn_check_errors(basis)
     _, C64, _ = oracle.compress_fwd(inp["X"], inp["ids"], inp["tok_emb"], inp["U"], n,
                                     pos_emb=inp["pos_emb"], pos=pos)
-    assert rel_fro(host(C), C64) <= TOL[dtype]
+    assert_parity(host(C), C64, dtype)
     _, X64, _ = oracle.decompress_fwd(host(C), inp["ids"], inp["tok_emb"], inp["U"], n,
                                       pos_emb=inp["pos_emb"], pos=pos)
-    assert rel_fro(host(Xr), X64) <= TOL[dtype]
+    assert_parity(host(Xr), X64, dtype)
     _, C64, _ = oracle.compress_fwd(inp["X"], inp["ids"], inp["tok_emb"], inp["U"], n)
-    assert rel_fro(host(C2), C64) <= TOL[dtype]
+    assert_parity(host(C2), C64, dtype)
     _, X64, _ = oracle.decompress_fwd(host(C2), inp["ids"], inp["tok_emb"], inp["U"], n)
-    assert rel_fro(host(Xr2), X64) <= TOL[dtype]
+    assert_parity(host(Xr2), X64, dtype)
     basis.destroy()
 
 
@@ -154,7 +154,7 @@ def test_bad_ids_zero_rows_and_report(sn, oracle, dtype):
     _, C64, st = oracle.compress_fwd(inp["X"], ids, inp["tok_emb"], inp["U"], n,
                                      pos_emb=inp["pos_emb"])
     assert st == 4
-    assert rel_fro(Ch, C64) <= TOL[dtype]
+    assert_parity(Ch, C64, dtype)
     Xr = sn.sn_decompress_fwd(basis, C, dev(ids), tok, n, pos_emb=pe)
     with pytest.raises(sn.SNError):
         sn.sn_check_errors(basis)
@@ -185,7 +185,7 @@ def test_project_weight(sn, oracle, dtype, d, k, cols, ld):
     sn.sn_project_weight(basis, Wd, out=out)
     sn.sn_check_errors(basis)
     _, W64, _ = oracle.project_weight(np.ascontiguousarray(Wh[:, :cols]), U)
-    assert rel_fro(host(out), W64) <= TOL[dtype]
+    assert_parity(host(out), W64, dtype)
     if cols < ld:      # the padding columns beyond `cols` are untouched
         assert bool((out_full[:, cols:] == 7.0).all())
     # in place, on a strided view with the same leading dimension
@@ -226,12 +226,12 @@ def test_projection_identities(sn, dtype):
         (0.02 * rng.standard_normal((d, cols))).astype(np.float32)
     W1 = sn.sn_project_weight(basis, dev(Wh))
     W2 = sn.sn_project_weight(basis, W1)
-    assert rel_fro(host(W2), widen(host(W1))) <= TOL[dtype]
+    assert_parity(host(W2), widen(host(W1)), dtype)
     B = rng.standard_normal((k, cols))
     In = U64 @ B
     Inh = W.to_bf16(In) if dtype == "bf16" else In.astype(np.float32)
     Pin = sn.sn_project_weight(basis, dev(Inh))
-    assert rel_fro(host(Pin), widen(Inh)) <= 2 * TOL[dtype]
+    assert_parity(host(Pin), widen(Inh), dtype, scale=2)
     basis.destroy()
 
 
@@ -356,9 +356,9 @@ def test_more_tiles_than_sms(sn, oracle, layout):
     _, C64, st = oracle.compress_fwd(inp["X"], inp["ids"], inp["tok_emb"], inp["U"], n,
                                      pos_emb=inp["pos_emb"])
     assert st == 0
-    assert rel_fro(host(C), C64) <= TOL["bf16"]
+    assert_parity(host(C), C64, "bf16")
     _, Cg64, _ = oracle.compress_bwd(inp["G"], inp["U"])
-    assert rel_fro(host(Cg), Cg64) <= TOL["bf16"]
+    assert_parity(host(Cg), Cg64, "bf16")
     # every row is covered: no row of C left at the guard fill or zero
     assert np.all(np.abs(widen(host(C))).sum(axis=1) > 0)
     basis.destroy()
@@ -401,18 +401,18 @@ def test_split_last_round(sn, oracle, layout):
     _, C64, st = oracle.compress_fwd(inp["X"], ids, inp["tok_emb"], inp["U"], n,
                                      pos_emb=inp["pos_emb"])
     assert st == 4
-    assert rel_fro(Ch, C64) <= TOL["bf16"]
+    assert_parity(Ch, C64, "bf16")
     good = np.setdiff1d(np.arange(T), bad)
     assert np.all(np.abs(widen(Ch[good])).sum(axis=1) > 0)
     _, Cg64, _ = oracle.compress_bwd(inp["G"], inp["U"])
-    assert rel_fro(host(Cg), Cg64) <= TOL["bf16"]
+    assert_parity(host(Cg), Cg64, "bf16")
     # the projected-table compress over the same tiles
     TU, PU = sn.sn_project_tables(basis, tok, pos_emb=pe)
     Cp = sn.sn_compress_fwd_projected(basis, X, dev(ids), TU, n, PU=PU)
     with pytest.raises(sn.SNError):
         sn.sn_check_errors(basis)
     assert np.all(widen(host(Cp)[bad]) == 0)
-    assert rel_fro(host(Cp), C64) <= TOL["bf16"]
+    assert_parity(host(Cp), C64, "bf16")
     if layout == "ragged":
         # explicit positions (not one contiguous run per tile: gathered rows)
         pos = np.random.default_rng(4).integers(0, n, T).astype(np.int32)
@@ -420,7 +420,7 @@ def test_split_last_round(sn, oracle, layout):
         sn.sn_check_errors(basis)
         _, C64, _ = oracle.compress_fwd(inp["X"], inp["ids"], inp["tok_emb"], inp["U"], n,
                                         pos_emb=inp["pos_emb"], pos=pos)
-        assert rel_fro(host(C), C64) <= TOL["bf16"]
+        assert_parity(host(C), C64, "bf16")
     basis.destroy()
 
 

@@ -11,7 +11,7 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_util import TOL, dev, host, rel_fro, widen
+from gpu_util import assert_parity, dev, host, widen
 from paper_2506_01260_gb300 import workloads as W
 
 pytestmark = pytest.mark.gpu
@@ -32,18 +32,18 @@ def test_tables_and_projected_compress(sn, oracle, T, n, d, k, vocab):
     # the tables: fp32 products of the bf16 tables with U (U rounded once to bf16)
     _, TU64, _ = oracle.compress_bwd(inp["tok_emb"], inp["U"])
     _, PU64, _ = oracle.compress_bwd(inp["pos_emb"], inp["U"])
-    assert rel_fro(TU.cpu().numpy(), TU64) <= TOL["bf16"]
-    assert rel_fro(PU.cpu().numpy(), PU64) <= TOL["bf16"]
+    assert_parity(TU.cpu().numpy(), TU64, "bf16")
+    assert_parity(PU.cpu().numpy(), PU64, "bf16")
     # the compress: the same C as the definition
     C = sn.sn_compress_fwd_projected(basis, X, ids, TU, n, PU=PU)
     sn.sn_check_errors(basis)
     _, C64, st = oracle.compress_fwd(inp["X"], inp["ids"], inp["tok_emb"], inp["U"], n,
                                      pos_emb=inp["pos_emb"])
     assert st == 0
-    assert rel_fro(host(C), C64) <= TOL["bf16"]
+    assert_parity(host(C), C64, "bf16")
     # and the same C as the d-wide kernel, within the bf16 bar
     Cd = sn.sn_compress_fwd(basis, X, ids, tok, n, pos_emb=pe)
-    assert rel_fro(host(C), widen(host(Cd))) <= TOL["bf16"]
+    assert_parity(host(C), widen(host(Cd)), "bf16")
     basis.destroy()
 
 
@@ -62,9 +62,9 @@ def test_projected_without_positions_and_with_explicit_positions(sn, oracle):
     sn.sn_check_errors(basis)
     _, C64, _ = oracle.compress_fwd(inp["X"], inp["ids"], inp["tok_emb"], inp["U"], n,
                                     pos_emb=inp["pos_emb"], pos=pos)
-    assert rel_fro(host(C1), C64) <= TOL["bf16"]
+    assert_parity(host(C1), C64, "bf16")
     _, C64, _ = oracle.compress_fwd(inp["X"], inp["ids"], inp["tok_emb"], inp["U"], n)
-    assert rel_fro(host(C2), C64) <= TOL["bf16"]
+    assert_parity(host(C2), C64, "bf16")
     basis.destroy()
 
 
@@ -85,7 +85,7 @@ def test_projected_bad_ids_zero_rows(sn, oracle):
                                     pos_emb=inp["pos_emb"])
     keep = np.ones(T, bool)
     keep[[5, 250]] = False
-    assert rel_fro(c[keep], C64[keep]) <= TOL["bf16"]
+    assert_parity(c[keep], C64[keep], "bf16")
     basis.destroy()
 
 
@@ -97,7 +97,7 @@ def test_build_ts(sn, oracle, vocab, d, k):
     sn.sn_check_errors(basis)
     _, TU64, _ = oracle.compress_bwd(inp["tok_emb"], inp["U"])
     _, TS64, _ = oracle.decompress_bwd(TU64, inp["U"])     # T_fixed U U^T in fp64
-    assert rel_fro(host(TS), TS64) <= TOL["bf16"]
+    assert_parity(host(TS), TS64, "bf16")
     basis.destroy()
 
 

@@ -7,7 +7,7 @@ tensor memory) matches the oracle."""
 import pytest
 import torch
 
-from gpu_util import TOL, dev, host, rel_fro
+from gpu_util import assert_parity, dev, host
 from paper_2506_01260_gb300 import workloads as W
 
 pytestmark = pytest.mark.gpu
@@ -40,11 +40,11 @@ def test_expired_wait_reports_timeout_and_context_survives(sn, oracle):
     _, C64, st = oracle.compress_fwd(inp["X"], inp["ids"], inp["tok_emb"], inp["U"], n,
                                      pos_emb=inp["pos_emb"])
     assert st == 0
-    assert rel_fro(host(C), C64) <= TOL["bf16"]
+    assert_parity(host(C), C64, "bf16")
     X64, st = oracle.decompress_fwd(host(C), inp["ids"], inp["tok_emb"], inp["U"], n,
                                     pos_emb=inp["pos_emb"])[1:]
     assert st == 0
-    assert rel_fro(host(Xr), X64) <= TOL["bf16"]
+    assert_parity(host(Xr), X64, "bf16")
     basis.destroy()
 
 
