@@ -7,13 +7,13 @@ batch and the bytes the method would send.  Top-k and sign quantization are
 kernels of the library; the low-rank comparator is a randomized rank-r
 factorisation X ~ Q B of the whole batch (sketch X Om with a Gaussian Om,
 power iterations, orthonormal Q of the sketch, B^T = X^T Q), composed of the
-library's contraction, accumulation and expansion calls, with the [T, r]
-sketch orthonormalised by CholeskyQR2 (fp64 Gram matrices); it sends Q and B,
-(T + d) r values.
+library's contraction, accumulation and expansion calls.  The [T, r] sketch is
+orthonormalised by the library too: the Grassmann step's retraction is
+CholeskyQR2 of U - eta * (step), so with eta = 0 it returns the orthonormal
+factor Q of its input (diag(R) > 0); it sends Q and B, (T + d) r values.
 """
 import math
 
-import numpy as np
 import torch
 
 from . import sn
@@ -45,11 +45,11 @@ def lowrank_roundtrip(X, r, power_iters=1, seed=0):
     b_om = sn.Basis(om)
 
     def orth(Y):
-        # CholeskyQR2: fp64 Gram products on the GPU, the r x r factor on the host
-        Q = Y.double()
-        for _ in range(2):
-            L = np.linalg.cholesky((Q.t() @ Q).cpu().numpy())
-            Q = Q @ torch.from_numpy(np.linalg.inv(L).T.copy()).to(Q.device)
+        # the Grassmann step's CholeskyQR2 retraction of Y itself (no step: eta = 0)
+        Yf = Y.float().contiguous()
+        b_y = sn.Basis(Yf)
+        Q = sn.sn_grassmann_step(b_y, torch.zeros_like(Yf), 1, 0.0)
+        b_y.destroy()
         return Q.to(torch.bfloat16).contiguous()
 
     def xt_times(Q):                                   # X^T Q, fp32 [d, r]
