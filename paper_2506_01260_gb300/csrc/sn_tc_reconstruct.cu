@@ -16,11 +16,12 @@
 //              read; the warp then stores its 32 rows with one TMA store and
 //              frees the embedding stage once the store has read them;
 //   warps 10-13 write each item's C rows into one of two TMEM A buffers (a
-//              thread per row, zero-padded to a multiple of 16), then fill the
-//              ring of embedding stages: per half block, the T_fixed rows of
-//              the tile's ids (and the positional rows when positions are not
-//              one contiguous run) with 16-byte cp.async copies into swizzled
-//              positions, or the positional tile with one TMA load.  Each
+//              thread per row, zero-padded to a multiple of 16; 4-byte loads
+//              when k is even), then fill the ring of embedding stages: per
+//              half block, the T_fixed rows of the tile's ids (and the
+//              positional rows when positions are not one contiguous run) with
+//              16-byte cp.async copies into swizzled positions, or the
+//              positional tile with one TMA load.  Each
 //              thread hands its copies to the stage's barrier
 //              (cp.async.mbarrier.arrive), which completes when all of them
 //              have landed, so the gather warps never wait for their own copies
@@ -31,6 +32,8 @@
 // in TMEM, shared memory is left to the two rings.
 // Each CTA walks an item's blocks starting at its own offset, so the CTAs'
 // B-operand reads are spread over the L2 instead of converging on one slice.
+// The ids (and positions) of the next item are loaded while the current one
+// is processed, so an item's start waits only for its C rows.
 // Every wait is bounded (SN_EBIT_TIMEOUT); an aborting CTA drains its copies
 // and MMAs and frees TMEM before it returns.
 #include "sn_tc.cuh"
@@ -189,23 +192,35 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
         const int row = 32 * q + lane;
         uint32_t g = 0;
         bool ok = true;
+        // the id (and position) of this thread's row, loaded an item ahead so
+        // that an item's start does not wait for them
+        int nid = 0, npos = 0;
+        auto load_row = [&](int item_) {
+            nid = 0;
+            npos = 0;
+            if (item_ < nitems) {
+                const int64_t t = tile_row0(item_ / p.chunks, p.reorder, p.batches, p.seq_len) + row;
+                if (t < p.rows) {
+                    nid = p.ids[t];
+                    if (p.has_pe && p.has_pos)
+                        npos = p.pos[t];
+                }
+            }
+        };
+        load_row(blockIdx.x);
         for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x) {
             const int tile = item / p.chunks, ch = item % p.chunks;
             const int blk0 = ch * p.bpi, blk1 = min(blk0 + p.bpi, p.nblk);
             const int64_t r0 = tile_row0(tile, p.reorder, p.batches, p.seq_len);
+            const int id = nid, ps = npos;
+            load_row(item + gridDim.x);
             bool bad = false;
-            {
-                const int64_t t = r0 + row;
-                if (t < p.rows) {
-                    const int id = p.ids[t];
-                    bad = id < 0 || id >= p.vocab;
-                    if (p.has_pe && p.has_pos) {
-                        const int ps = p.pos[t];
-                        bad = bad || ps < 0 || ps >= p.seq_len;
-                    }
-                    if (bad && ch == 0)
-                        atomicOr(p.err, SN_EBIT_BAD_ID);
-                }
+            if (r0 + row < p.rows) {
+                bad = id < 0 || id >= p.vocab;
+                if (p.has_pe && p.has_pos)
+                    bad = bad || ps < 0 || ps >= p.seq_len;
+                if (bad && ch == 0)
+                    atomicOr(p.err, SN_EBIT_BAD_ID);
             }
             for (int j = 0; j < blk1 - blk0 && ok; ++j, ++g) {
                 const int blk = block_at(blk0, blk1, j);
@@ -283,10 +298,35 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
             tma_prefetch(&p.mapPE);
         uint32_t g = 0, e = 0, it = 0;
         bool ok = true;
+        // ids and positions of this thread's 8 gather rows, loaded an item ahead
+        int nid[8], npos[8];
+        auto load_rows = [&](int item_) {
+            const int64_t q0 = item_ < nitems
+                                   ? tile_row0(item_ / p.chunks, p.reorder, p.batches, p.seq_len)
+                                   : p.rows;
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int64_t t = q0 + (tt >> 3) + 16 * u;
+                nid[u] = 0;
+                npos[u] = 0;
+                if (t < p.rows) {
+                    nid[u] = p.ids[t];
+                    if (p.has_pe && p.has_pos)
+                        npos[u] = p.pos[t];
+                }
+            }
+        };
+        load_rows(blockIdx.x);
         for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++it) {
             const int tile = item / p.chunks, ch = item % p.chunks;
             const int blk0 = ch * p.bpi, blk1 = min(blk0 + p.bpi, p.nblk);
             const int64_t r0 = tile_row0(tile, p.reorder, p.batches, p.seq_len);
+            int cid[8], cpos[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                cid[u] = nid[u];
+                cpos[u] = npos[u];
+            }
             {
                 // A operand: row arow of the tile's C rows, two bf16 per TMEM
                 // column, zero past k (and for rows past the end)
@@ -300,14 +340,21 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
                 const unsigned short *crow = (const unsigned short *)p.C + t * p.k;
                 const uint32_t a_tmem = tmem + ((uint32_t)(32 * (warp & 3)) << 16) + kReconACol +
                                         ab * kReconAStride;
+                const uint32_t *crow32 = (const uint32_t *)(p.C + t * p.k);   // k even: 4-byte aligned
                 for (int w0 = 0; w0 < 8 * p.kmma; w0 += 16) {
                     uint32_t h[16];
+                    if ((p.k & 1) == 0) {
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        const int j0 = 2 * (w0 + i);
-                        const uint32_t lo = (t < p.rows && j0 < p.k) ? __ldg(crow + j0) : 0u;
-                        const uint32_t hi = (t < p.rows && j0 + 1 < p.k) ? __ldg(crow + j0 + 1) : 0u;
-                        h[i] = lo | (hi << 16);
+                        for (int i = 0; i < 16; ++i)
+                            h[i] = (t < p.rows && 2 * (w0 + i) < p.k) ? __ldg(crow32 + w0 + i) : 0u;
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) {
+                            const int j0 = 2 * (w0 + i);
+                            const uint32_t lo = (t < p.rows && j0 < p.k) ? __ldg(crow + j0) : 0u;
+                            const uint32_t hi = (t < p.rows && j0 + 1 < p.k) ? __ldg(crow + j0 + 1) : 0u;
+                            h[i] = lo | (hi << 16);
+                        }
                     }
                     tmem_st16(a_tmem + w0, h);
                 }
@@ -317,6 +364,7 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
                 if (lane == 0)
                     mbar_arrive(afull_b + 8 * ab);
             }
+            load_rows(item + gridDim.x);
             const bool pe_tile = p.has_pe && !p.has_pos && (r0 % p.seq_len) + BM <= p.seq_len;
             // element offsets of this thread's 8 rows in T_fixed and P (invalid
             // ids / positions read row 0; the epilogue zeroes those rows)
@@ -326,11 +374,11 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
                 const int64_t t = r0 + (tt >> 3) + 16 * u;
                 int64_t id = 0, ps = 0;
                 if (t < p.rows) {
-                    id = p.ids[t];
+                    id = cid[u];
                     if (id < 0 || id >= p.vocab)
                         id = 0;
                     if (p.has_pe) {
-                        ps = p.has_pos ? (int64_t)p.pos[t] : t % p.seq_len;
+                        ps = p.has_pos ? (int64_t)cpos[u] : t % p.seq_len;
                         if (ps < 0 || ps >= p.seq_len)
                             ps = 0;
                     }
