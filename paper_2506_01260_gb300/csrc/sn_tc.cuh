@@ -99,6 +99,58 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
     return ok != 0;
 }
 
+// Relaxed forms for a role that, after a wait, only issues copies into a buffer
+// another role has released and reads nothing that role published: a relaxed
+// wait or arrival does not hold the thread until its own earlier loads have
+// returned, so loads issued ahead (the next work item's ids and C rows) stay
+// in flight across it.
+__device__ __forceinline__ void mbar_arrive_relaxed(uint32_t bar)
+{
+    asm volatile("mbarrier.arrive.relaxed.cta.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_tx_relaxed(uint32_t bar, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.relaxed.cta.shared::cta.b64 _, [%0], %1;" ::"r"(bar),
+                 "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ bool mbar_test_relaxed(uint32_t bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{ .reg .pred p; mbarrier.try_wait.parity.relaxed.cta.shared::cta.b64 p, [%1], %2; "
+        "selp.u32 %0, 1, 0, p; }"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// warp_wait with a relaxed poll by lane 0 alone (the other lanes observe
+// nothing themselves).  All 32 lanes must call it.
+__device__ __forceinline__ bool warp_wait_relaxed(uint32_t bar, uint32_t parity,
+                                                  volatile int *abort, unsigned int *err)
+{
+    int ok = 1;
+    if ((threadIdx.x & 31) == 0 && !mbar_test_relaxed(bar, parity)) {
+        const uint64_t t0 = global_ns();
+        while (true) {
+            if (mbar_test_relaxed(bar, parity))
+                break;
+            if (*abort) {
+                ok = 0;
+                break;
+            }
+            if (global_ns() - t0 > kWaitLimitNs) {
+                *abort = 1;
+                atomicOr(err, SN_EBIT_TIMEOUT);
+                ok = 0;
+                break;
+            }
+        }
+    }
+    return __shfl_sync(0xffffffffu, ok, 0) != 0;
+}
+
 // Short bounded wait used only while draining after an abort.
 __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity)
 {
@@ -379,6 +431,32 @@ __device__ __forceinline__ void gather_tile_async(uint32_t dst, const __nv_bfloa
 }
 
 
+// A 4-byte load issued where it is written: an asm volatile statement keeps its
+// place among the other volatile statements, so a load meant to be in flight
+// ahead of its use is not moved down to the use.
+__device__ __forceinline__ int ld_issue(const int *p)
+{
+    int v;
+    asm volatile("ld.global.nc.b32 %0, [%1];" : "=r"(v) : "l"(p));
+    return v;
+}
+
+// gather_tile_async with the 8 rows given as row indices of a table whose rows
+// are row_len elements long
+__device__ __forceinline__ void gather_rows_async(uint32_t dst, const __nv_bfloat16 *table,
+                                                  const int (&rows)[8], int64_t col0,
+                                                  int64_t row_len, int tt)
+{
+    const int c = tt & 7;
+    const int64_t col = col0 + 8 * c;
+    const bool in = col + 8 <= row_len;       // row_len is a multiple of 8
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+        const int r = (tt >> 3) + 16 * u;
+        cp_async16(dst + sw128(r, c), table + (int64_t)rows[u] * row_len + (in ? col : 0),
+                   in ? 16u : 0u);
+    }
+}
 
 }  // namespace tc
 }  // namespace sn

@@ -17,7 +17,8 @@
 //              frees the embedding stage once the store has read them;
 //   warps 10-13 write each item's C rows into one of two TMEM A buffers (a
 //              thread per row, zero-padded to a multiple of 16; 4-byte loads
-//              when k is even), then fill the ring of embedding stages: per
+//              when k is even), the next item's during the current item's
+//              last half blocks, and fill the ring of embedding stages: per
 //              half block, the T_fixed rows of the tile's ids (and the
 //              positional rows when positions are not one contiguous run) with
 //              16-byte cp.async copies into swizzled positions, or the
@@ -32,8 +33,13 @@
 // in TMEM, shared memory is left to the two rings.
 // Each CTA walks an item's blocks starting at its own offset, so the CTAs'
 // B-operand reads are spread over the L2 instead of converging on one slice.
-// The ids (and positions) of the next item are loaded while the current one
-// is processed, so an item's start waits only for its C rows.
+// An item's start costs the gather warps, the pipeline's bottleneck, almost
+// nothing: the next item's ids (and positions) are loaded and turned into
+// row indices a few half blocks into the current item, and its A operand is
+// loaded a chunk at a time over the current item's last half blocks; the
+// gather warps' own waits and arrivals on the embedding ring are relaxed
+// (they publish nothing and read nothing the epilogue wrote), so none of
+// them holds a warp until those loads have returned.
 // Every wait is bounded (SN_EBIT_TIMEOUT); an aborting CTA drains its copies
 // and MMAs and frees TMEM before it returns.
 #include "sn_tc.cuh"
@@ -44,6 +50,12 @@ namespace tc {
 namespace {
 
 constexpr int NB = BN_WIDE;
+// half blocks between the loads of one chunk of the next item's A and its
+// write to TMEM (about the time a load spends behind the copies in flight)
+constexpr int kAPreDist = 10;
+// half block of an item at which the next item's gather rows are prepared
+// (their ids were loaded at half block 1)
+constexpr int kRowsPrep = 6;
 constexpr uint32_t kTmemCols = 512;
 static_assert(kReconAcc * NB <= (int)kReconACol && kReconACol + 2 * kReconAStride <= kTmemCols,
               "TMEM plan");
@@ -298,36 +310,86 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
             tma_prefetch(&p.mapPE);
         uint32_t g = 0, e = 0, it = 0;
         bool ok = true;
-        // ids and positions of this thread's 8 gather rows, loaded an item ahead
-        int nid[8], npos[8];
-        auto load_rows = [&](int item_) {
-            const int64_t q0 = item_ < nitems
-                                   ? tile_row0(item_ / p.chunks, p.reorder, p.batches, p.seq_len)
-                                   : p.rows;
+        // The next item's gather rows (this thread's 8 rows of T_fixed and P)
+        // are prepared during the current item, where the gather warps wait for
+        // free stages anyway: its ids and positions are loaded after the
+        // item's first half block and turned into row indices a few half
+        // blocks later, so an item starts with its first copies.
+        int nrow_t[8], nrow_p[8];
+        bool npe_tile = false;
+        int64_t nq0 = p.rows;
+        auto load_rows = [&](int tile_) {
+            nq0 = tile_ >= 0 ? tile_row0(tile_, p.reorder, p.batches, p.seq_len) : p.rows;
 #pragma unroll
             for (int u = 0; u < 8; ++u) {
-                const int64_t t = q0 + (tt >> 3) + 16 * u;
-                nid[u] = 0;
-                npos[u] = 0;
+                const int64_t t = nq0 + (tt >> 3) + 16 * u;
+                nrow_t[u] = 0;
+                nrow_p[u] = 0;
                 if (t < p.rows) {
-                    nid[u] = p.ids[t];
+                    nrow_t[u] = ld_issue(p.ids + t);
                     if (p.has_pe && p.has_pos)
-                        npos[u] = p.pos[t];
+                        nrow_p[u] = ld_issue(p.pos + t);
                 }
             }
         };
-        load_rows(blockIdx.x);
-        for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++it) {
-            const int tile = item / p.chunks, ch = item % p.chunks;
-            const int blk0 = ch * p.bpi, blk1 = min(blk0 + p.bpi, p.nblk);
-            const int64_t r0 = tile_row0(tile, p.reorder, p.batches, p.seq_len);
-            int cid[8], cpos[8];
+        // ids / positions -> row indices (invalid ones read row 0; the epilogue
+        // zeroes those rows); positional rows only where they are gathered
+        auto prep_rows = [&]() {
+            const int base = p.has_pe && !p.has_pos ? (int)(nq0 % p.seq_len) : 0;
+            npe_tile = p.has_pe && !p.has_pos && base + BM <= p.seq_len;
 #pragma unroll
             for (int u = 0; u < 8; ++u) {
-                cid[u] = nid[u];
-                cpos[u] = npos[u];
+                const int off = (tt >> 3) + 16 * u;
+                const bool in = nq0 + off < p.rows;
+                int id = nrow_t[u];
+                if (!in || id < 0 || id >= p.vocab)
+                    id = 0;
+                nrow_t[u] = id;
+                int ps = 0;
+                if (p.has_pe && !npe_tile && in) {
+                    ps = p.has_pos ? nrow_p[u] : (base + off) % p.seq_len;
+                    if (ps < 0 || ps >= p.seq_len)
+                        ps = 0;
+                }
+                nrow_p[u] = ps;
             }
-            {
+        };
+        // 16 words (32 bf16 of C) of row t of A, zero past k and past the end
+        auto load_a = [&](int64_t t, int w0, uint32_t (&h)[16]) {
+            const unsigned short *crow = (const unsigned short *)p.C + t * p.k;
+            const uint32_t *crow32 = (const uint32_t *)(p.C + t * p.k);   // k even: 4-byte aligned
+            if ((p.k & 1) == 0) {
+#pragma unroll
+                for (int i = 0; i < 16; ++i)
+                    h[i] = (t < p.rows && 2 * (w0 + i) < p.k) ? __ldg(crow32 + w0 + i) : 0u;
+            } else {
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    const int j0 = 2 * (w0 + i);
+                    const uint32_t lo = (t < p.rows && j0 < p.k) ? __ldg(crow + j0) : 0u;
+                    const uint32_t hi = (t < p.rows && j0 + 1 < p.k) ? __ldg(crow + j0 + 1) : 0u;
+                    h[i] = lo | (hi << 16);
+                }
+            }
+        };
+        const uint32_t a_lane = tmem + ((uint32_t)(32 * (warp & 3)) << 16) + kReconACol;
+        const int nch = (8 * p.kmma + 15) / 16;    // 16-word chunks of a row of A
+        load_rows((int)blockIdx.x < nitems ? (int)blockIdx.x / p.chunks : -1);
+        prep_rows();
+        bool a_ready = false;      // this item's A was written during the previous item
+        for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++it) {
+            const int ch = item % p.chunks;
+            const int blk0 = ch * p.bpi, blk1 = min(blk0 + p.bpi, p.nblk);
+            const int64_t r0 = nq0;
+            const bool pe_tile = npe_tile;
+            const int pe_row0 = pe_tile ? (int)(r0 % p.seq_len) : 0;
+            int trow[8], prow[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                trow[u] = nrow_t[u];
+                prow[u] = nrow_p[u];
+            }
+            if (!a_ready) {
                 // A operand: row arow of the tile's C rows, two bf16 per TMEM
                 // column, zero past k (and for rows past the end)
                 const uint32_t ab = it & 1;
@@ -336,27 +398,10 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
                     break;
                 }
                 tc_fence_after();
-                const int64_t t = r0 + arow;
-                const unsigned short *crow = (const unsigned short *)p.C + t * p.k;
-                const uint32_t a_tmem = tmem + ((uint32_t)(32 * (warp & 3)) << 16) + kReconACol +
-                                        ab * kReconAStride;
-                const uint32_t *crow32 = (const uint32_t *)(p.C + t * p.k);   // k even: 4-byte aligned
-                for (int w0 = 0; w0 < 8 * p.kmma; w0 += 16) {
+                for (int m = 0; m < nch; ++m) {
                     uint32_t h[16];
-                    if ((p.k & 1) == 0) {
-#pragma unroll
-                        for (int i = 0; i < 16; ++i)
-                            h[i] = (t < p.rows && 2 * (w0 + i) < p.k) ? __ldg(crow32 + w0 + i) : 0u;
-                    } else {
-#pragma unroll
-                        for (int i = 0; i < 16; ++i) {
-                            const int j0 = 2 * (w0 + i);
-                            const uint32_t lo = (t < p.rows && j0 < p.k) ? __ldg(crow + j0) : 0u;
-                            const uint32_t hi = (t < p.rows && j0 + 1 < p.k) ? __ldg(crow + j0 + 1) : 0u;
-                            h[i] = lo | (hi << 16);
-                        }
-                    }
-                    tmem_st16(a_tmem + w0, h);
+                    load_a(r0 + arow, 16 * m, h);
+                    tmem_st16(a_lane + ab * kReconAStride + 16 * m, h);
                 }
                 tmem_st_wait();
                 tc_fence_before();
@@ -364,33 +409,42 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
                 if (lane == 0)
                     mbar_arrive(afull_b + 8 * ab);
             }
-            load_rows(item + gridDim.x);
-            const bool pe_tile = p.has_pe && !p.has_pos && (r0 % p.seq_len) + BM <= p.seq_len;
-            // element offsets of this thread's 8 rows in T_fixed and P (invalid
-            // ids / positions read row 0; the epilogue zeroes those rows)
-            int64_t trow[8], prow[8];
-#pragma unroll
-            for (int u = 0; u < 8; ++u) {
-                const int64_t t = r0 + (tt >> 3) + 16 * u;
-                int64_t id = 0, ps = 0;
-                if (t < p.rows) {
-                    id = cid[u];
-                    if (id < 0 || id >= p.vocab)
-                        id = 0;
-                    if (p.has_pe) {
-                        ps = p.has_pos ? (int64_t)cpos[u] : t % p.seq_len;
-                        if (ps < 0 || ps >= p.seq_len)
-                            ps = 0;
-                    }
-                }
-                trow[u] = id * p.ncols;
-                prow[u] = ps * p.ncols;
-            }
+            const bool has_next = item + (int)gridDim.x < nitems;
+            const int next_tile = has_next ? (item + (int)gridDim.x) / p.chunks : -1;
+            // The next item's A goes into the other A buffer while this item's
+            // last nch * kAPreDist half blocks are issued: chunk m is loaded at
+            // half block nh - (nch - m) kAPreDist and written to TMEM one
+            // distance later, so its loads are in flight behind the copies
+            // already queued instead of holding up the next item's start.
+            const int nh = 2 * (blk1 - blk0);
+            const bool pre = has_next && nh >= nch * kAPreDist;
+            const uint32_t nab = (it + 1) & 1;
+            const int64_t nt = (has_next ? tile_row0(next_tile, p.reorder, p.batches, p.seq_len) : 0) + arow;
+            uint32_t ha[16];
+            int mq = 0, hq = 0;
             for (int j = 0; j < blk1 - blk0 && ok; ++j, ++g) {
                 const int blk = block_at(blk0, blk1, j);
-                for (int hh = 0; hh < 2; ++hh, ++e) {
+                for (int hh = 0; hh < 2; ++hh, ++e, ++hq) {
+                    if (hq == 1)
+                        load_rows(next_tile);
+                    else if (hq == kRowsPrep)
+                        prep_rows();
+                    if (pre && hq == nh - (nch - mq) * kAPreDist) {
+                        if (mq == 0) {
+                            if (!warp_wait_relaxed(aempty_b + 8 * nab, (((it + 1) >> 1) & 1) ^ 1,
+                                                   abort_flag, p.err)) {
+                                ok = false;
+                                break;
+                            }
+                            tc_fence_after();
+                        } else {
+                            tmem_st16(a_lane + nab * kReconAStride + 16 * (mq - 1), ha);
+                        }
+                        load_a(nt, 16 * mq, ha);
+                        ++mq;
+                    }
                     const uint32_t es = e % SE;
-                    if (!warp_wait(eempty_b + 8 * es, ((e / SE) & 1) ^ 1, abort_flag, p.err)) {
+                    if (!warp_wait_relaxed(eempty_b + 8 * es, ((e / SE) & 1) ^ 1, abort_flag, p.err)) {
                         ok = false;
                         break;
                     }
@@ -399,18 +453,35 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
                     if (tt == 0) {
                         const uint32_t pb = efull_b + 8 * es;
                         if (pe_tile) {
-                            mbar_arrive_tx(pb, kTile);
-                            tma_load_2d(tb + pl.t_bytes, &p.mapPE, col0, (int)(r0 % p.seq_len), pb);
+                            mbar_arrive_tx_relaxed(pb, kTile);
+                            tma_load_2d(tb + pl.t_bytes, &p.mapPE, col0, pe_row0, pb);
                         } else {
-                            mbar_arrive(pb);
+                            mbar_arrive_relaxed(pb);
                         }
                     }
-                    gather_tile_async(tb, p.tok, trow, col0, p.ncols, tt);
+                    gather_rows_async(tb, p.tok, trow, col0, p.ncols, tt);
                     if (p.has_pe && !pe_tile)
-                        gather_tile_async(tb + pl.t_bytes, p.pe, prow, col0, p.ncols, tt);
+                        gather_rows_async(tb + pl.t_bytes, p.pe, prow, col0, p.ncols, tt);
                     cp_async_arrive(efull_b + 8 * es);
                 }
             }
+            // items too short to reach those half blocks
+            if (nh <= 1)
+                load_rows(next_tile);
+            if (nh <= kRowsPrep)
+                prep_rows();
+            if (pre) {
+                if (mq > 0)
+                    tmem_st16(a_lane + nab * kReconAStride + 16 * (mq - 1), ha);
+                tmem_st_wait();
+                if (ok) {
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0)
+                        mbar_arrive_relaxed(afull_b + 8 * nab);
+                }
+            }
+            a_ready = pre && ok;
         }
         cp_async_wait0();
         // positional tiles still in flight after an abort
