@@ -24,7 +24,10 @@
 //              positions; each thread hands its copies to the stage's barrier
 //              (cp.async.mbarrier.arrive), so the gather warps never wait for
 //              their own copies, and the MMA thread fences toward the async
-//              proxy after the barrier completes.
+//              proxy after the barrier completes.  The next item's ids are
+//              loaded and turned into row indices during the current item,
+//              and the gather warps' waits for free stages are relaxed, so an
+//              item's first copies wait for no load.
 // Each CTA walks an item's chunks starting at its own offset, so the CTAs' U^T
 // reads are spread over the L2 instead of converging on one slice.
 // Every wait is bounded; a wait that expires raises SN_EBIT_TIMEOUT and the
@@ -35,6 +38,10 @@
 namespace sn {
 namespace tc {
 namespace {
+
+// chunk of an item at which the gather warps prepare the next item's rows
+// (their ids were loaded at chunk 1)
+constexpr int kRowsPrep = 6;
 
 // j-th chunk of an item: every CTA starts at a different chunk so that the
 // CTAs do not all read the same U^T chunk from one L2 slice at once.
@@ -333,45 +340,88 @@ __global__ void __launch_bounds__(contract_threads(MODE), 1)
         const int tt = threadIdx.x - 192;    // 0..127
         uint32_t g = 0;
         bool ok = true;
-        for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x) {
-            const ItemSpan sp = item_span(p, item);
-            const int tile = sp.tile, kc0 = sp.kc0, kc1 = sp.kc1;
-            const int64_t r0 = tile_row0(tile, p.reorder, p.batches, p.seq_len);
-            const bool pe_tile = p.has_pe && !p.has_pos && (r0 % p.seq_len) + BM <= p.seq_len;
-            // element offsets of this thread's 8 rows in T_fixed and P (invalid
-            // ids / positions read row 0; the epilogue zeroes those rows)
-            int64_t trow[8], prow[8];
+        // The next item's gather rows (this thread's 8 rows of T_fixed and P)
+        // are prepared during the current item, where the gather warps wait for
+        // free stages anyway: its ids and positions are loaded after the
+        // item's first chunk and turned into row indices a few chunks later,
+        // so an item starts with its first copies.
+        int nrow_t[8], nrow_p[8];
+        bool npe_tile = false;
+        int64_t nq0 = p.rows;
+        auto load_rows = [&](int tile_) {
+            nq0 = tile_ >= 0 ? tile_row0(tile_, p.reorder, p.batches, p.seq_len) : p.rows;
 #pragma unroll
             for (int u = 0; u < 8; ++u) {
-                const int64_t t = r0 + (tt >> 3) + 16 * u;
-                int64_t id = 0, ps = 0;
+                const int64_t t = nq0 + (tt >> 3) + 16 * u;
+                nrow_t[u] = 0;
+                nrow_p[u] = 0;
                 if (t < p.rows) {
-                    id = p.ids[t];
-                    if (id < 0 || id >= p.vocab)
-                        id = 0;
-                    if (p.has_pe) {
-                        ps = p.has_pos ? (int64_t)p.pos[t] : t % p.seq_len;
-                        if (ps < 0 || ps >= p.seq_len)
-                            ps = 0;
-                    }
+                    nrow_t[u] = ld_issue(p.ids + t);
+                    if (p.has_pe && p.has_pos)
+                        nrow_p[u] = ld_issue(p.pos + t);
                 }
-                trow[u] = id * p.d;
-                prow[u] = ps * p.d;
             }
-            for (int j = 0; j < kc1 - kc0; ++j, ++g) {
+        };
+        // ids / positions -> row indices (invalid ones read row 0; the epilogue
+        // zeroes those rows); positional rows only where they are gathered
+        auto prep_rows = [&]() {
+            const int base = p.has_pe && !p.has_pos ? (int)(nq0 % p.seq_len) : 0;
+            npe_tile = p.has_pe && !p.has_pos && base + BM <= p.seq_len;
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int off = (tt >> 3) + 16 * u;
+                const bool in = nq0 + off < p.rows;
+                int id = nrow_t[u];
+                if (!in || id < 0 || id >= p.vocab)
+                    id = 0;
+                nrow_t[u] = id;
+                int ps = 0;
+                if (p.has_pe && !npe_tile && in) {
+                    ps = p.has_pos ? nrow_p[u] : (base + off) % p.seq_len;
+                    if (ps < 0 || ps >= p.seq_len)
+                        ps = 0;
+                }
+                nrow_p[u] = ps;
+            }
+        };
+        load_rows((int)blockIdx.x < nitems ? item_span(p, blockIdx.x).tile : -1);
+        prep_rows();
+        for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x) {
+            const ItemSpan sp = item_span(p, item);
+            const int kc0 = sp.kc0, kc1 = sp.kc1;
+            const bool pe_tile = npe_tile;
+            int trow[8], prow[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                trow[u] = nrow_t[u];
+                prow[u] = nrow_p[u];
+            }
+            const int next_tile =
+                item + (int)gridDim.x < nitems ? item_span(p, item + gridDim.x).tile : -1;
+            const int nj = kc1 - kc0;
+            for (int j = 0; j < nj; ++j, ++g) {
+                if (j == 1)
+                    load_rows(next_tile);
+                else if (j == kRowsPrep)
+                    prep_rows();
                 const int kc = chunk_at(kc0, kc1, j);
                 const int s = g % S;
                 const uint32_t n = g / S;
-                if (!warp_wait(empty_b + 8 * s, (n & 1) ^ 1, abort_flag, p.err)) {
+                if (!warp_wait_relaxed(empty_b + 8 * s, (n & 1) ^ 1, abort_flag, p.err)) {
                     ok = false;
                     break;
                 }
                 const uint32_t tb = base + s * pl.stage_bytes + pl.a_bytes + pl.u_bytes;
-                gather_tile_async(tb, p.tok, trow, (int64_t)kc * BK, p.d, tt);
+                gather_rows_async(tb, p.tok, trow, (int64_t)kc * BK, p.d, tt);
                 if (p.has_pe && !pe_tile)
-                    gather_tile_async(tb + pl.raw_bytes, p.pe, prow, (int64_t)kc * BK, p.d, tt);
+                    gather_rows_async(tb + pl.raw_bytes, p.pe, prow, (int64_t)kc * BK, p.d, tt);
                 cp_async_arrive(full_b + 8 * s);
             }
+            // items too short to reach those chunks
+            if (nj <= 1)
+                load_rows(next_tile);
+            if (nj <= kRowsPrep)
+                prep_rows();
         }
         cp_async_wait0();
     }
