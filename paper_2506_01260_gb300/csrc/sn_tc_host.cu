@@ -100,6 +100,17 @@ void recon_stages(int katoms, int has_pe, int *sb, int *se)
     *se = s;
 }
 
+// Paired reconstruction: two B stages of 64 U rows, as many 48 KB embedding
+// stages as fit (at most 12).
+void pair_stages(int katoms, int *sb, int *se)
+{
+    *sb = 2;
+    int s = 12;
+    while (s > 2 && pair_plan(katoms, *sb, s).total > kSmemLimit)
+        --s;
+    *se = s;
+}
+
 // Tiles ordered position-block-major when every sequence of the batch shares
 // the same positional rows in whole 128-row blocks.
 void tile_order(int64_t T, int seq_len, bool has_pe, bool has_pos, int *reorder, int *batches)
@@ -461,6 +472,16 @@ cudaError_t tc_decompress(const sn_basis &b, const TcArgs &a, __nv_bfloat16 *X_o
     p.ntiles = (int)((a.T + BM - 1) / BM);
     split_blocks(p.ntiles, p.nblk, sms, &p.bpi, &p.chunks);
     tile_order(a.T, a.seq_len, has_pe, p.has_pos, &p.reorder, &p.batches);
+    if (a.gather && has_pe && p.reorder && p.batches % 2 == 0 && b.d % nb == 0 && b.n_pad <= 128) {
+        // sequences 2i and 2i + 1 add the same positional tiles: one work item
+        // covers both tiles of a pair (p.ntiles counts pairs), U in 64-row boxes
+        if (!map2d(&p.mapA, b.up16, b.k64, b.d, (uint64_t)b.k64 * 2, 64, 64, true))
+            return cudaErrorInvalidValue;
+        p.ntiles /= 2;
+        split_blocks(p.ntiles, p.nblk, sms, &p.bpi, &p.chunks);
+        pair_stages(p.katoms, &p.stages, &p.estages);
+        return launch_reconstruct_pair(p, std::min(p.ntiles * p.chunks, sms), s);
+    }
     const int grid = std::min(p.ntiles * p.chunks, sms);
     if (a.gather) {
         recon_stages(p.katoms, has_pe, &p.stages, &p.estages);

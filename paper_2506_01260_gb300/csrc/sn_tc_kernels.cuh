@@ -196,6 +196,37 @@ __host__ __device__ inline ReconPlan recon_plan(int katoms, int has_pe, int sb, 
 // (one per half block), warps 10-13 A operand and row gathers
 constexpr int kReconThreads = 448;
 
+// The paired reconstruction (two row tiles that add the same positional tile):
+// per 64-column half block, one B stage of 64 U rows and one embedding stage of
+// both tiles' [128 x 64] T_fixed tiles and their one positional tile.  TMEM
+// holds two accumulator slots of 128 columns (the half block of each tile side
+// by side) and two A buffers of both tiles' C rows.
+constexpr int kPairAcc = 2;               // accumulator slots of 2 x 64 columns
+constexpr uint32_t kPairACol = 256;       // first TMEM column of the A buffers
+
+struct PairPlan {
+    uint32_t b_bytes, e_bytes, bar_off, total;
+};
+
+__host__ __device__ inline PairPlan pair_plan(int katoms, int sb, int se)
+{
+    PairPlan p;
+    p.b_bytes = (uint32_t)katoms * 64 * 128;
+    p.e_bytes = 3 * kTile;
+    p.bar_off = (uint32_t)sb * p.b_bytes + (uint32_t)se * p.e_bytes;
+    p.total = p.bar_off + 8 * (2 * sb + 2 * se + 2 * kPairAcc + 5) + 16 + 1024;
+    return p;
+}
+
+// First row of the first tile of pair `pp`: pairs run position-block-major
+// over sequences (0, 1), (2, 3), ... of a batch of `batches` (even) sequences of
+// seq_len rows; the pair's second tile starts seq_len rows later.
+__host__ __device__ inline int64_t pair_row0(int pp, int batches, int seq_len)
+{
+    const int half = batches >> 1;
+    return (int64_t)(2 * (pp % half)) * seq_len + (int64_t)(pp / half) * BM;
+}
+
 // Row tile -> first row.  With `reorder`, tiles run position-block-major so the
 // b sequences of a batch that share positional rows are processed together
 // and the positional table is read from HBM once.
@@ -214,6 +245,7 @@ cudaError_t launch_contract(int mode, const ContractParams &p, int grid, cudaStr
 cudaError_t launch_expand(int amode, const ExpandParams &p, int grid, cudaStream_t s,
                           bool dependent = false);
 cudaError_t launch_reconstruct(const ExpandParams &p, int grid, cudaStream_t s);
+cudaError_t launch_reconstruct_pair(const ExpandParams &p, int grid, cudaStream_t s);
 
 }  // namespace tc
 }  // namespace sn
