@@ -215,6 +215,38 @@ def test_project_weight_in_place_full_size(sn, d, k, cols):
     basis.destroy()
 
 
+def test_project_weight_repeated_and_very_wide(sn, oracle):
+    """The first pass writes fp32 partials over several d-ranges per column tile
+    into the caller's workspace and the second sums them: calls with other
+    column counts in between give identical results, and a W of 4097 column
+    tiles (half a million columns) matches the oracle."""
+    d, k = 2048, 41                         # 32 chunks of d: several splits per tile
+    rng = np.random.default_rng(17)
+    U = W.orthonormal_basis(d, k, rng).astype(np.float32)
+    basis = sn.Basis(dev(U))
+    g = torch.Generator(device="cuda").manual_seed(5)
+    Wa = (0.02 * torch.randn(d, 1000, generator=g, device="cuda")).to(torch.bfloat16)
+    Wb = (0.02 * torch.randn(d, 304, generator=g, device="cuda")).to(torch.bfloat16)
+    ref = sn.sn_project_weight(basis, Wa)
+    for _ in range(3):
+        sn.sn_project_weight(basis, Wb)
+        assert torch.equal(sn.sn_project_weight(basis, Wa), ref)
+    sn.sn_check_errors(basis)
+    _, W64, _ = oracle.project_weight(host(Wa), U)
+    assert_parity(host(ref), W64, "bf16")
+    basis.destroy()
+    # 4097 tiles of 128 columns
+    d, k, cols = 64, 8, 4097 * 128
+    U = W.orthonormal_basis(d, k, rng).astype(np.float32)
+    basis = sn.Basis(dev(U))
+    Wh = W.to_bf16(0.02 * rng.standard_normal((d, cols)))
+    out = sn.sn_project_weight(basis, dev(Wh))
+    sn.sn_check_errors(basis)
+    _, W64, _ = oracle.project_weight(Wh, U)
+    assert_parity(host(out), W64, "bf16")
+    basis.destroy()
+
+
 @pytest.mark.parametrize("dtype", DTYPES)
 def test_projection_identities(sn, dtype):
     """P^2 = P and P U = U on the GPU output (Sec. 4.3; U^T U = I, App. A)."""
