@@ -18,7 +18,8 @@
 //   warps 10-13 write each item's C rows into one of two TMEM A buffers (a
 //              thread per row, zero-padded to a multiple of 16; 4-byte loads
 //              when k is even), the next item's during the current item's
-//              last half blocks, and fill the ring of embedding stages: per
+//              last half blocks (the first item's are written by the idle
+//              epilogue warps), and fill the ring of embedding stages: per
 //              half block, the T_fixed rows of the tile's ids (and the
 //              positional rows when positions are not one contiguous run) with
 //              16-byte cp.async copies into swizzled positions, or the
@@ -76,6 +77,28 @@ __device__ __forceinline__ uint32_t add_emb(float a0, float a1, uint32_t pe, uin
     return pack_bf16(add_bf16_lo(te, add_bf16_lo(pe, a0)), add_bf16_hi(te, add_bf16_hi(pe, a1)));
 }
 
+// 16 words (32 bf16) of C row t from word w0 on, zero past k and past the end;
+// 4-byte loads when k is even (rows 4-byte aligned), 2-byte loads otherwise
+__device__ __forceinline__ void load_c_words(const ExpandParams &p, int64_t t, int w0,
+                                             uint32_t (&h)[16])
+{
+    const unsigned short *crow = (const unsigned short *)p.C + t * p.k;
+    const uint32_t *crow32 = (const uint32_t *)(p.C + t * p.k);
+    if ((p.k & 1) == 0) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i)
+            h[i] = (t < p.rows && 2 * (w0 + i) < p.k) ? __ldg(crow32 + w0 + i) : 0u;
+    } else {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            const int j0 = 2 * (w0 + i);
+            const uint32_t lo = (t < p.rows && j0 < p.k) ? __ldg(crow + j0) : 0u;
+            const uint32_t hi = (t < p.rows && j0 + 1 < p.k) ? __ldg(crow + j0 + 1) : 0u;
+            h[i] = lo | (hi << 16);
+        }
+    }
+}
+
 __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_constant__ ExpandParams p)
 {
     extern __shared__ uint8_t smem_raw[];
@@ -113,7 +136,9 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
             mbar_init(acce_b + 8 * b, 8);     // both epilogue groups
         }
         for (int b = 0; b < 2; ++b) {
-            mbar_init(afull_b + 8 * b, 4);    // the four gather warps
+            // the eight epilogue warps (the first item), or the four gather
+            // warps arriving twice each (every later item)
+            mbar_init(afull_b + 8 * b, 8);
             mbar_init(aempty_b + 8 * b, 1);
         }
         mbar_init(drain_b, 1);
@@ -224,6 +249,28 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
             }
         };
         load_row(blockIdx.x);
+        if ((int)blockIdx.x < nitems) {
+            // The first item's A operand: the epilogue warps are idle until the
+            // first accumulator, so they write it (group g the 16-word chunks
+            // m = g, g + 2) while the gather warps start their copies.
+            const int nch = (8 * p.kmma + 15) / 16;
+            const int64_t t = tile_row0((int)blockIdx.x / p.chunks, p.reorder, p.batches, p.seq_len) + row;
+            uint32_t h[2][16];
+#pragma unroll
+            for (int i = 0; i < 2; ++i)
+                if (grp + 2 * i < nch)
+                    load_c_words(p, t, 16 * (grp + 2 * i), h[i]);
+            const uint32_t a_lane = tmem + ((uint32_t)(32 * q) << 16) + kReconACol;
+#pragma unroll
+            for (int i = 0; i < 2; ++i)
+                if (grp + 2 * i < nch)
+                    tmem_st16(a_lane + 16 * (grp + 2 * i), h[i]);
+            tmem_st_wait();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(afull_b);              // A buffer 0
+        }
         for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x) {
             const int tile = item / p.chunks, ch = item % p.chunks;
             const int blk0 = ch * p.bpi, blk1 = min(blk0 + p.bpi, p.nblk);
@@ -358,29 +405,13 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
                 nrow_p[u] = ps;
             }
         };
-        // 16 words (32 bf16 of C) of row t of A, zero past k and past the end
-        auto load_a = [&](int64_t t, int w0, uint32_t (&h)[16]) {
-            const unsigned short *crow = (const unsigned short *)p.C + t * p.k;
-            const uint32_t *crow32 = (const uint32_t *)(p.C + t * p.k);   // k even: 4-byte aligned
-            if ((p.k & 1) == 0) {
-#pragma unroll
-                for (int i = 0; i < 16; ++i)
-                    h[i] = (t < p.rows && 2 * (w0 + i) < p.k) ? __ldg(crow32 + w0 + i) : 0u;
-            } else {
-#pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    const int j0 = 2 * (w0 + i);
-                    const uint32_t lo = (t < p.rows && j0 < p.k) ? __ldg(crow + j0) : 0u;
-                    const uint32_t hi = (t < p.rows && j0 + 1 < p.k) ? __ldg(crow + j0 + 1) : 0u;
-                    h[i] = lo | (hi << 16);
-                }
-            }
-        };
         const uint32_t a_lane = tmem + ((uint32_t)(32 * (warp & 3)) << 16) + kReconACol;
         const int nch = (8 * p.kmma + 15) / 16;    // 16-word chunks of a row of A
         load_rows((int)blockIdx.x < nitems ? (int)blockIdx.x / p.chunks : -1);
         prep_rows();
-        bool a_ready = false;      // this item's A was written during the previous item
+        // this item's A is written (the first item's by the epilogue warps,
+        // later ones during the previous item)
+        bool a_ready = true;
         for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++it) {
             const int ch = item % p.chunks;
             const int blk0 = ch * p.bpi, blk1 = min(blk0 + p.bpi, p.nblk);
@@ -404,14 +435,14 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
                 tc_fence_after();
                 for (int m = 0; m < nch; ++m) {
                     uint32_t h[16];
-                    load_a(r0 + arow, 16 * m, h);
+                    load_c_words(p, r0 + arow, 16 * m, h);
                     tmem_st16(a_lane + ab * kReconAStride + 16 * m, h);
                 }
                 tmem_st_wait();
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0)
-                    mbar_arrive(afull_b + 8 * ab);
+                    mbar_arrive_cnt(afull_b + 8 * ab, 2);
             }
             const bool has_next = item + (int)gridDim.x < nitems;
             const int next_tile = has_next ? (item + (int)gridDim.x) / p.chunks : -1;
@@ -444,7 +475,7 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
                         } else {
                             tmem_st16(a_lane + nab * kReconAStride + 16 * (mq - 1), ha);
                         }
-                        load_a(nt, 16 * mq, ha);
+                        load_c_words(p, nt, 16 * mq, ha);
                         ++mq;
                     }
                     const uint32_t es = e % SE;
@@ -482,7 +513,7 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
                     tc_fence_before();
                     __syncwarp();
                     if (lane == 0)
-                        mbar_arrive_relaxed(afull_b + 8 * nab);
+                        mbar_arrive_cnt_relaxed(afull_b + 8 * nab, 2);
                 }
             }
             a_ready = pre && ok;
@@ -502,28 +533,6 @@ __global__ void __launch_bounds__(kReconThreads, 1) k_reconstruct(const __grid_c
     }
 }
 
-
-// 16 words (32 bf16) of C row t from word w0 on, zero past k and past the end;
-// 4-byte loads when k is even (rows 4-byte aligned), 2-byte loads otherwise
-__device__ __forceinline__ void load_c_words(const ExpandParams &p, int64_t t, int w0,
-                                             uint32_t (&h)[16])
-{
-    const unsigned short *crow = (const unsigned short *)p.C + t * p.k;
-    const uint32_t *crow32 = (const uint32_t *)(p.C + t * p.k);
-    if ((p.k & 1) == 0) {
-#pragma unroll
-        for (int i = 0; i < 16; ++i)
-            h[i] = (t < p.rows && 2 * (w0 + i) < p.k) ? __ldg(crow32 + w0 + i) : 0u;
-    } else {
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-            const int j0 = 2 * (w0 + i);
-            const uint32_t lo = (t < p.rows && j0 < p.k) ? __ldg(crow + j0) : 0u;
-            const uint32_t hi = (t < p.rows && j0 + 1 < p.k) ? __ldg(crow + j0 + 1) : 0u;
-            h[i] = lo | (hi << 16);
-        }
-    }
-}
 
 // ---------------------------------------------------------------------------------
 // The paired form.  When every sequence of the batch covers the same positions in

@@ -6,7 +6,8 @@ and 2i + 1 at one position block together (they add the same positional tile).
 Checked against the fp64 oracle: k from 1 to 128 (odd and even k, one to four
 16-word chunks of A per tile), widths of one to eight 128-column blocks, more
 work items than SMs (several items per CTA, so the next item's operands are
-prepared during the current one), invalid ids, and C = 0, where the output is
+prepared during the current one, or written at the item's start when the items
+are short), invalid ids, and C = 0, where the output is
 round(T_fixed[id] + P[pos]) bit for bit.  The same batch with the positions
 given explicitly runs the single-tile kernel; both kernels compute the same
 fp32 sums and must agree bit for bit.
@@ -71,6 +72,28 @@ def test_paired_more_items_than_sms(sn, oracle):
     sn.sn_check_errors(basis)
     assert guards_intact(fullX)
     _, X64, st = oracle.decompress_fwd(host(C), inp["ids"], inp["tok_emb"], inp["U"], n,
+                                       pos_emb=inp["pos_emb"])
+    assert st == 0
+    assert_parity(host(Xr), X64, "bf16")
+    basis.destroy()
+
+
+def test_paired_short_items_write_a_at_item_start(sn, oracle):
+    """k = 128 (four chunks of A per tile) and items of two blocks: an item is
+    too short to load the next item's eight chunks during it, so every later
+    item's A is written by the gather warps at the item's start."""
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    nseq, n, d, k, vocab = 2 * (sms + 8), 128, 256, 128, 900
+    T = nseq * n
+    inp = inputs("pairs_short", nseq, n, d, k, vocab, seed=7)
+    basis = sn.Basis(dev(inp["U"]))
+    C = np.asarray(W.to_bf16(np.random.default_rng(7).standard_normal((T, k))))
+    fullX, Xr = guarded((T, d), torch.bfloat16)
+    sn.sn_decompress_fwd(basis, dev(C), dev(inp["ids"]), dev(inp["tok_emb"]), n,
+                         pos_emb=dev(inp["pos_emb"]), out=Xr)
+    sn.sn_check_errors(basis)
+    assert guards_intact(fullX)
+    _, X64, st = oracle.decompress_fwd(C, inp["ids"], inp["tok_emb"], inp["U"], n,
                                        pos_emb=inp["pos_emb"])
     assert st == 0
     assert_parity(host(Xr), X64, "bf16")
