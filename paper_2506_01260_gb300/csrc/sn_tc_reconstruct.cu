@@ -687,7 +687,7 @@ __global__ void __launch_bounds__(kReconThreads, 1)
                     }
                 }
                 if (ok)
-                    mma_commit(aempty_b + 8 * ab);       // both A buffers of the item free
+                    mma_commit(aempty_b + 8 * ab);       // the item's A buffer (both tiles) free
             }
             if (!ok) {
                 mma_commit(drain_b);
