@@ -155,3 +155,43 @@ def test_paired_equals_single_tile_kernel(sn, k):
     sn.sn_check_errors(basis)
     assert np.array_equal(host(Xp), host(Xs))
     basis.destroy()
+
+
+def _sweep_cases():
+    """Seeded small shapes on both sides of the pairing conditions."""
+    rng = np.random.default_rng(2024)
+    cases = []
+    for i in range(16):
+        nseq = int(rng.integers(1, 7))                 # odd counts run the single-tile kernel
+        n = int(rng.choice([128, 256, 384, 200]))      # 200: not a whole number of tiles
+        d = int(rng.choice([128, 256, 384, 520]))      # 520: not a whole number of blocks
+        k = int(rng.choice([1, 7, 16, 41, 64, 96, 128]))
+        k = min(k, d)
+        explicit = bool(rng.integers(0, 4) == 0)       # explicit positions: single-tile kernel
+        cases.append((i, nseq, n, d, k, explicit))
+    return cases
+
+
+@pytest.mark.parametrize("case", _sweep_cases(), ids=lambda c: "s%d_b%d_n%d_d%d_k%d%s" % (
+    c[0], c[1], c[2], c[3], c[4], "_pos" if c[5] else ""))
+def test_reconstruction_shape_sweep(sn, oracle, case):
+    """Paired and single-tile reconstructions against the oracle over seeded
+    shapes (even and odd sequence counts, lengths and widths on and off the
+    tile and block sizes, explicit positions)."""
+    i, nseq, n, d, k, explicit = case
+    T = nseq * n
+    inp = inputs("sweep%d" % i, nseq, n, d, k, 700, seed=100 + i)
+    basis = sn.Basis(dev(inp["U"]))
+    C = np.asarray(W.to_bf16(np.random.default_rng(i).standard_normal((T, k))))
+    pos = (np.arange(T) % n).astype(np.int32) if explicit else None
+    fullX, Xr = guarded((T, d), torch.bfloat16)
+    sn.sn_decompress_fwd(basis, dev(C), dev(inp["ids"]), dev(inp["tok_emb"]), n,
+                         pos_emb=dev(inp["pos_emb"]), pos=None if pos is None else dev(pos),
+                         out=Xr)
+    sn.sn_check_errors(basis)
+    assert guards_intact(fullX)
+    _, X64, st = oracle.decompress_fwd(C, inp["ids"], inp["tok_emb"], inp["U"], n,
+                                       pos_emb=inp["pos_emb"], pos=pos)
+    assert st == 0
+    assert_parity(host(Xr), X64, "bf16")
+    basis.destroy()
